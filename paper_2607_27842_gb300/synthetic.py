@@ -1,0 +1,203 @@
+"""Seeded synthetic workloads shaped like the paper's backbones.
+
+Holds none of the method's arithmetic: model shapes, schedules, site lists,
+random-init weights N(0, 0.02) and conditioning inputs only.  Both the CUDA
+path and the CPU oracle consume what this module produces.
+
+The five workloads (stand-ins for the paper's DiT-XL/2 on ImageNet-256,
+FLUX.1-dev and Qwen-Image on DrawBench and HunyuanVideo-1.5 on VBench,
+whose checkpoints and datasets are not used):
+  tiny     4-block class-conditional DiT, fp32, 8x8x4 latent, 10 Euler steps
+  dit_xl2  DiT-XL/2 shape, bf16, 32x32x4 latent, batch 8 (16 with guidance), 50 DDIM steps
+  flux     19 dual + 38 single MMDiT blocks, 4096 image + 512 text tokens, 50 Euler steps
+  qwen     60 dual MMDiT blocks, 4096 image + 256 text tokens, guidance, 50 Euler steps
+  hunyuan  54 dual MMDiT blocks, 9x30x53 video tokens + 256 text, 3-D rotary, 50 Euler steps
+"""
+
+import dataclasses
+
+import numpy as np
+
+from .featfix import weight_spec
+
+WEIGHT_STD = 0.02
+
+
+@dataclasses.dataclass(frozen=True)
+class ModelShape:
+    name: str
+    arch: str            # "dit" | "mmdit"
+    n_dual: int          # DiT blocks, or MMDiT two-stream blocks
+    n_single: int
+    hidden: int
+    heads: int
+    head_dim: int
+    mlp: int
+    in_ch: int
+    out_ch: int
+    patch: int
+    patch_t: int
+    lat_f: int           # 0 for images
+    lat_h: int
+    lat_w: int
+    txt_tokens: int
+    n_classes: int
+    batch: int           # latent samples
+    cfg: bool            # model batch = [cond ; uncond]
+    cfg_scale: float
+    rope_dims: int
+    dtype: str           # "f32" | "bf16"
+    sampler: str         # "euler" | "ddim"
+
+    @property
+    def n_layers(self):
+        return self.n_dual + self.n_single
+
+    @property
+    def batch_model(self):
+        return self.batch * (2 if self.cfg else 1)
+
+    @property
+    def img_tokens(self):
+        gf = self.lat_f // self.patch_t if self.lat_f > 0 else 1
+        return gf * (self.lat_h // self.patch) * (self.lat_w // self.patch)
+
+    @property
+    def tokens(self):
+        return self.img_tokens + self.txt_tokens
+
+    @property
+    def latent_dims(self):
+        f = (self.lat_f,) if self.lat_f > 0 else ()
+        return (self.batch, self.in_ch) + f + (self.lat_h, self.lat_w)
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    shape: ModelShape
+    steps: int
+    K: int
+    refresh: tuple
+    sites: tuple         # (step, layer) pairs
+
+
+def refresh_every(steps, interval):
+    """Fixed-interval full refresh: steps 0, interval, 2 * interval, ..."""
+    return tuple(range(0, steps, interval))
+
+
+def diagonal_sites(steps, L, refresh, n_sites):
+    """A fixed, spread-out site set: site j at layer floor((j + 1/2) L / n) and
+    at the non-refresh step of rank floor((j + 1/2) |M| / n)."""
+    rs = set(refresh)
+    M = [i for i in range(steps) if i not in rs]
+    out = []
+    for j in range(n_sites):
+        layer = (2 * j + 1) * L // (2 * n_sites)
+        step = M[(2 * j + 1) * len(M) // (2 * n_sites)]
+        out.append((step, layer))
+    return tuple(out)
+
+
+def _shape(**kw):
+    base = dict(n_single=0, patch_t=1, lat_f=0, txt_tokens=0, n_classes=0, cfg=False, cfg_scale=4.0,
+                rope_dims=0)
+    base.update(kw)
+    return ModelShape(**base)
+
+
+SHAPES = {
+    "tiny": _shape(name="tiny", arch="dit", n_dual=4, hidden=128, heads=4, head_dim=32, mlp=512, in_ch=4,
+                   out_ch=4, patch=1, lat_h=8, lat_w=8, n_classes=10, batch=1, dtype="f32", sampler="euler"),
+    "dit_xl2": _shape(name="dit_xl2", arch="dit", n_dual=28, hidden=1152, heads=16, head_dim=72, mlp=4608,
+                      in_ch=4, out_ch=8, patch=2, lat_h=32, lat_w=32, n_classes=1000, batch=8, cfg=True,
+                      dtype="bf16", sampler="ddim"),
+    "flux": _shape(name="flux", arch="mmdit", n_dual=19, n_single=38, hidden=3072, heads=24, head_dim=128,
+                   mlp=12288, in_ch=16, out_ch=16, patch=2, lat_h=128, lat_w=128, txt_tokens=512, batch=1,
+                   rope_dims=2, dtype="bf16", sampler="euler"),
+    "qwen": _shape(name="qwen", arch="mmdit", n_dual=60, hidden=3072, heads=24, head_dim=128, mlp=12288, in_ch=16,
+                   out_ch=16, patch=2, lat_h=128, lat_w=128, txt_tokens=256, batch=1, cfg=True, rope_dims=2,
+                   dtype="bf16", sampler="euler"),
+    "hunyuan": _shape(name="hunyuan", arch="mmdit", n_dual=54, hidden=2048, heads=16, head_dim=128, mlp=8192,
+                      in_ch=16, out_ch=16, patch=2, patch_t=1, lat_f=9, lat_h=60, lat_w=106, txt_tokens=256,
+                      batch=1, rope_dims=3, dtype="bf16", sampler="euler"),
+}
+
+
+def workload(name):
+    """The schedule of each workload: draft order, refresh interval, sites."""
+    s = SHAPES[name]
+    if name == "tiny":
+        return Workload(s, 10, 1, (0, 3, 6, 9), ((4, 2), (7, 1)))
+    cfg = {"dit_xl2": (50, 2, 5, 8), "flux": (50, 1, 6, 12), "qwen": (50, 2, 5, 16), "hunyuan": (50, 1, 5, 12)}
+    steps, K, every, n_sites = cfg[name]
+    ref = refresh_every(steps, every)
+    return Workload(s, steps, K, ref, diagonal_sites(steps, s.n_layers, ref, n_sites))
+
+
+def reduced(shape, **overrides):
+    """A smaller variant of a shape (fewer blocks, smaller latent, ...)."""
+    return dataclasses.replace(shape, **overrides)
+
+
+# ----------------------------------------------------------------------------
+# tensors (torch: CPU or CUDA)
+# ----------------------------------------------------------------------------
+
+def torch_dtype(shape):
+    import torch
+    return torch.float32 if shape.dtype == "f32" else torch.bfloat16
+
+
+def make_weights(shape, seed=0, device="cpu", names=None):
+    """Random-init weights: every tensor N(0, 0.02) from its own seeded
+    generator (seed * 1000003 + index), stored in the model dtype.
+    ``names`` restricts generation to a subset (same values)."""
+    import torch
+    out = {}
+    want = None if names is None else set(names)
+    for idx, (name, dims) in enumerate(weight_spec(shape)):
+        if want is not None and name not in want:
+            continue
+        g = torch.Generator(device=device)
+        g.manual_seed(seed * 1000003 + idx)
+        t = torch.randn(dims, generator=g, device=device, dtype=torch.float32) * WEIGHT_STD
+        out[name] = t.to(torch_dtype(shape)).contiguous()
+    return out
+
+
+def make_cond(shape, seed=2, device="cpu"):
+    """DiT: int32 labels [B_model] (uniform classes; the guidance half uses the
+    null class n_classes).  MMDiT: float32 text tokens [B_model, N_txt, C]
+    from N(0, 1) (the guidance half from seed + 1000)."""
+    import torch
+    g = torch.Generator(device="cpu")
+    g.manual_seed(seed)
+    if shape.arch == "dit":
+        lab = torch.randint(0, shape.n_classes, (shape.batch,), generator=g, dtype=torch.int64)
+        if shape.cfg:
+            lab = torch.cat([lab, torch.full((shape.batch,), shape.n_classes, dtype=torch.int64)])
+        return lab.to(torch.int32).to(device)
+    txt = torch.randn((shape.batch, shape.txt_tokens, shape.hidden), generator=g, dtype=torch.float32)
+    if shape.cfg:
+        g2 = torch.Generator(device="cpu")
+        g2.manual_seed(seed + 1000)
+        unc = torch.randn((shape.batch, shape.txt_tokens, shape.hidden), generator=g2, dtype=torch.float32)
+        txt = torch.cat([txt, unc])
+    return txt.contiguous().to(device)
+
+
+def to_numpy64(t):
+    """float64 numpy copy of a torch tensor (bf16 values are exact in fp64)."""
+    import torch
+    return t.detach().to("cpu", torch.float64).numpy()
+
+
+def oracle_weights(weights):
+    return {k: to_numpy64(v) for k, v in weights.items()}
+
+
+def oracle_cond(shape, cond):
+    if shape.arch == "dit":
+        return np.asarray(cond.cpu().numpy(), dtype=np.int64)
+    return to_numpy64(cond)
