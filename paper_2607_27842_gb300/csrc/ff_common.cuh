@@ -1,0 +1,252 @@
+// Internal declarations shared by the FeatFix CUDA translation units.
+// Not part of the public ABI (include/featfix.h, include/featfix_ops.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+namespace ff {
+
+enum DType : int { F32 = 0, BF16 = 1 };
+typedef __nv_bfloat16 bf16;
+
+static inline int dsize(DType t) { return t == F32 ? 4 : 2; }
+
+// ---------------------------------------------------------------------------
+// element conversion and 16-byte vectors
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
+template <class T> __device__ __forceinline__ T from_f(float x);
+template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float x) { return __float2bfloat16_rn(x); }
+
+template <class T> struct VecN { static constexpr int n = 16 / (int)sizeof(T); };
+
+__device__ __forceinline__ void ld16(const float* p, float (&v)[4]) {
+  float4 q = *reinterpret_cast<const float4*>(p);
+  v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+}
+__device__ __forceinline__ void ld16(const bf16* p, float (&v)[8]) {
+  uint4 q = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float2 f = __bfloat1622float2(h[i]);
+    v[2 * i] = f.x;
+    v[2 * i + 1] = f.y;
+  }
+}
+__device__ __forceinline__ void st16(float* p, const float (&v)[4]) {
+  *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+}
+__device__ __forceinline__ void st16(bf16* p, const float (&v)[8]) {
+  uint4 q;
+  __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&q);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+  *reinterpret_cast<uint4*>(p) = q;
+}
+// round-trip through the storage type (value as it is stored)
+__device__ __forceinline__ float round_to(float x, float*) { return x; }
+__device__ __forceinline__ float round_to(float x, bf16*) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+__device__ __forceinline__ float gelu_tanh(float x) {
+  const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
+  return 0.5f * x * (1.0f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+}
+__device__ __forceinline__ float silu(float x) { return x / (1.0f + expf(-x)); }
+
+// ---------------------------------------------------------------------------
+// fused GEMM epilogue: y = act(acc + bias); rope; out = resid + gate * y;
+// hist_out = stored(out) - hist_base
+// ---------------------------------------------------------------------------
+struct EpiArgs {
+  const void* bias;      // [N] model dtype (nullable)
+  int act;               // 0 identity, 1 GELU(tanh)
+  int act_col0;          // activation only on columns >= act_col0
+  const float* gate;     // gate rows (nullable): gate[b * gate_stride + n]
+  int gate_stride;
+  int seg_split;         // batch of row r: r < seg_split ? r / rpb0 : (r - seg_split) / rpb1
+  int rpb0, rpb1;
+  const void* resid;     // [M, ld_resid] model dtype (nullable); out = resid + (gate ? gate*y : y)
+  int ld_resid;
+  void* out;             // [M, ldo]
+  int ldo;
+  int out_f32;           // out (and out2) are float32 instead of the model dtype
+  int split_col;         // columns >= split_col go to out2 at column n - split_col (N if unused)
+  void* out2;
+  int ldo2;
+  const void* hist_base; // [M, ldo] model dtype (nullable)
+  void* hist_out;        // [M, ldo] model dtype: stored(out) - hist_base
+  const float2* rope;    // (cos, sin) table [rope_period][rope_half] (nullable)
+  int rope_row0;         // rows >= rope_row0 are rotated
+  int rope_period;       // image tokens per sample
+  int rope_cols;         // columns < rope_cols (q and k) are rotated
+  int rope_hd;           // head width d (pairs (2j, 2j+1) within a head)
+};
+
+static inline EpiArgs epi_plain(void* out, int ldo) {
+  EpiArgs e = {};
+  e.out = out;
+  e.ldo = ldo;
+  e.act_col0 = 0;
+  e.split_col = 0x7fffffff;
+  e.rpb0 = 1;
+  e.rpb1 = 1;
+  return e;
+}
+
+__device__ __forceinline__ int epi_batch(const EpiArgs& e, int r) {
+  return r < e.seg_split ? r / e.rpb0 : (r - e.seg_split) / e.rpb1;
+}
+
+// Applies the epilogue to CH consecutive accumulator columns n0 .. n0+CH-1
+// of row m.  The chunk must not straddle split_col, act_col0 or rope_cols,
+// and CH must be a multiple of the 16-byte vector width of T.  Columns >= N
+// are skipped (N % vector width == 0).
+template <class T, int CH>
+__device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N, float (&v)[CH]) {
+  constexpr int V = VecN<T>::n;
+  if (e.bias) {
+    const T* b = reinterpret_cast<const T*>(e.bias);
+#pragma unroll
+    for (int j = 0; j < CH; j += V) {
+      if (n0 + j < N) {
+        float bb[V];
+        ld16(b + n0 + j, bb);
+#pragma unroll
+        for (int q = 0; q < V; ++q) v[j + q] += bb[q];
+      }
+    }
+  }
+  if (e.rope && m >= e.rope_row0 && n0 < e.rope_cols) {
+    const int tok = (m - e.rope_row0) % e.rope_period;
+    const int half = e.rope_hd >> 1;
+#pragma unroll
+    for (int j = 0; j < CH; j += 2) {
+      const int pair = ((n0 + j) % e.rope_hd) >> 1;
+      const float2 cs = e.rope[(size_t)tok * half + pair];
+      const float a = v[j], b = v[j + 1];
+      v[j] = a * cs.x - b * cs.y;
+      v[j + 1] = a * cs.y + b * cs.x;
+    }
+  }
+  if (e.act == 1 && n0 >= e.act_col0) {
+#pragma unroll
+    for (int j = 0; j < CH; ++j) v[j] = gelu_tanh(v[j]);
+  }
+  if (e.gate) {
+    const float* g = e.gate + (size_t)epi_batch(e, m) * e.gate_stride + n0;
+#pragma unroll
+    for (int j = 0; j < CH; j += 4) {
+      if (n0 + j < N) {
+        float4 gg = *reinterpret_cast<const float4*>(g + j);
+        v[j] *= gg.x; v[j + 1] *= gg.y; v[j + 2] *= gg.z; v[j + 3] *= gg.w;
+      }
+    }
+  }
+  if (e.resid) {
+    const T* rs = reinterpret_cast<const T*>(e.resid) + (size_t)m * e.ld_resid + n0;
+#pragma unroll
+    for (int j = 0; j < CH; j += V) {
+      if (n0 + j < N) {
+        float rr[V];
+        ld16(rs + j, rr);
+#pragma unroll
+        for (int q = 0; q < V; ++q) v[j + q] += rr[q];
+      }
+    }
+  }
+  const bool second = n0 >= e.split_col;
+  const int col = second ? n0 - e.split_col : n0;
+  const int ld = second ? e.ldo2 : e.ldo;
+  void* obase = second ? e.out2 : e.out;
+  if (e.out_f32) {
+    float* o = reinterpret_cast<float*>(obase) + (size_t)m * ld + col;
+#pragma unroll
+    for (int j = 0; j < CH; j += 4) {
+      if (n0 + j < N) {
+        float t[4] = {v[j], v[j + 1], v[j + 2], v[j + 3]};
+        st16(o + j, t);
+      }
+    }
+  } else {
+    T* o = reinterpret_cast<T*>(obase) + (size_t)m * ld + col;
+#pragma unroll
+    for (int j = 0; j < CH; j += V) {
+      if (n0 + j < N) {
+        float t[V];
+#pragma unroll
+        for (int q = 0; q < V; ++q) t[q] = v[j + q];
+        st16(o + j, t);
+      }
+    }
+  }
+  if (e.hist_out) {
+    const T* hb = reinterpret_cast<const T*>(e.hist_base) + (size_t)m * e.ldo + n0;
+    T* ho = reinterpret_cast<T*>(e.hist_out) + (size_t)m * e.ldo + n0;
+#pragma unroll
+    for (int j = 0; j < CH; j += V) {
+      if (n0 + j < N) {
+        float u[V], t[V];
+        ld16(hb + j, u);
+#pragma unroll
+        for (int q = 0; q < V; ++q) t[q] = round_to(v[j + q], (T*)nullptr) - u[q];
+        st16(ho + j, t);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// launchers (return the launch error; work is asynchronous on `s`)
+// ---------------------------------------------------------------------------
+struct Hist4 { const void* p[4]; };
+
+// Process-wide count of kernels this library has launched.
+void count_launches(long long n);
+long long launches_total();
+inline cudaError_t launched() {
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int nt, long long n, cudaStream_t s);
+size_t verify_workspace_bytes(long long n);
+cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
+                          int write_draft, double* sums, void* ws, cudaStream_t s);
+cudaError_t launch_ln_mod(DType dt, const void* x, void* out, long long rows, int C, const float* shift,
+                          const float* scale, int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s);
+cudaError_t launch_linear_small(DType wt, const float* x, int B, int K, const void* W, const void* bias, int N,
+                                float* y, int ldy, int silu_in, int silu_out, cudaStream_t s);
+cudaError_t launch_sinusoid(float t, float* out, int dim, cudaStream_t s);
+cudaError_t launch_cond_finish(DType wt, const float* e, const void* y_emb, const int* labels, int B, int C,
+                               float* c_out, float* csilu_out, cudaStream_t s);
+cudaError_t launch_patchify(DType dt, const float* latent, int B_lat, int B_model, int Cin, int F, int H, int W,
+                            int p, int pt, void* out, cudaStream_t s);
+cudaError_t launch_convert(DType dt, const float* in, void* out, long long n, cudaStream_t s);
+cudaError_t launch_sampler(const float* model_out, float* latent, int B_lat, int cfg, float cfg_scale, int Cin,
+                           int Cout, int F, int H, int W, int p, int pt, float c1, float c2, cudaStream_t s);
+cudaError_t launch_noise(unsigned long long seed, float* out, long long n, cudaStream_t s);
+cudaError_t launch_pos2d(DType dt, void* out, int B, int gh, int gw, int C, cudaStream_t s);
+
+// dense layers: out = epilogue(A[M,K] W[N,K]^T)
+cudaError_t gemm_simt(DType dt, int M, int N, int K, const void* A, int lda, const void* W, int ldw,
+                      const EpiArgs& e, cudaStream_t s);
+cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, int ldw, const EpiArgs& e,
+                    cudaStream_t s);
+unsigned int gemm_tc_watchdog_take();
+
+// attention over the token-row layout (see featfix_token_row)
+struct AttnArgs {
+  const void* q; const void* k; const void* v;  // base pointers (column offsets applied)
+  int ld_qkv;
+  void* out; int ld_out;
+  int B, Nt, Ni, H, hd;
+};
+cudaError_t attention(DType dt, const AttnArgs& a, cudaStream_t s);
+cudaError_t attention_simt(DType dt, const AttnArgs& a, cudaStream_t s);
+
+}  // namespace ff

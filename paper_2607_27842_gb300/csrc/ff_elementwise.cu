@@ -1,0 +1,556 @@
+// Bandwidth-bound kernels of the FeatFix denoising step: the draft (Eq. 2),
+// the fused paid check / forward (Eqs. 3-5), adaLN LayerNorm-modulation,
+// conditioning GEMVs, embedding, sampler update and the seeded latent.
+#include "ff_common.cuh"
+
+#include <cooperative_groups.h>
+#include <math.h>
+
+#include <atomic>
+
+namespace cg = cooperative_groups;
+
+namespace ff {
+
+static std::atomic<long long> g_launches{0};
+void count_launches(long long n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+long long launches_total() { return g_launches.load(std::memory_order_relaxed); }
+
+static int g_num_sms = 0;
+static int num_sms() {
+  if (g_num_sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (g_num_sms <= 0) g_num_sms = 148;
+  }
+  return g_num_sms;
+}
+
+// ---------------------------------------------------------------------------
+// Draft (Eq. 2, weight form): x <- x + sum_j w_j R_j.  One 16-byte vector per
+// thread per iteration, every operand streamed once, grid-stride over a grid
+// sized to a multiple of the SM count.
+// ---------------------------------------------------------------------------
+template <class T, int NT>
+__device__ __forceinline__ void draft_vec(const T* __restrict__ xu, const Hist4& h, const float (&w)[4], long long i,
+                                          float (&a)[VecN<T>::n]) {
+  constexpr int V = VecN<T>::n;
+  ld16(xu + i * V, a);
+#pragma unroll
+  for (int j = 0; j < NT; ++j) {
+    float r[V];
+    ld16(reinterpret_cast<const T*>(h.p[j]) + i * V, r);
+#pragma unroll
+    for (int q = 0; q < V; ++q) a[q] = __fmaf_rn(w[j], r[q], a[q]);
+  }
+}
+
+template <class T, int NT>
+__device__ __forceinline__ float draft_scalar(const T* xu, const Hist4& h, const float (&w)[4], long long i) {
+  float a = to_f(xu[i]);
+#pragma unroll
+  for (int j = 0; j < NT; ++j) a = __fmaf_rn(w[j], to_f(reinterpret_cast<const T*>(h.p[j])[i]), a);
+  return a;
+}
+
+template <class T, int NT>
+__global__ void __launch_bounds__(256) k_draft(T* __restrict__ x, Hist4 h, float w0, float w1, float w2, float w3,
+                                               long long n) {
+  constexpr int V = VecN<T>::n;
+  const float w[4] = {w0, w1, w2, w3};
+  const long long nvec = n / V;
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += stride) {
+    float a[V];
+    draft_vec<T, NT>(x, h, w, i, a);
+    st16(x + i * V, a);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < n - nvec * V) {
+    const long long i = nvec * V + threadIdx.x;
+    x[i] = from_f<T>(draft_scalar<T, NT>(x, h, w, i));
+  }
+}
+
+static int stream_grid(long long nvec, int threads) {
+  long long want = (nvec + threads - 1) / threads;
+  long long cap = (long long)num_sms() * 8;
+  if (want > cap) want = cap;
+  if (want < 1) want = 1;
+  return (int)want;
+}
+
+template <class T>
+static cudaError_t draft_t(void* x, const Hist4& h, const float* w, int nt, long long n, cudaStream_t s) {
+  const int grid = stream_grid(n / VecN<T>::n, 256);
+  T* xp = reinterpret_cast<T*>(x);
+  switch (nt) {
+    case 1: k_draft<T, 1><<<grid, 256, 0, s>>>(xp, h, w[0], w[1], w[2], w[3], n); break;
+    case 2: k_draft<T, 2><<<grid, 256, 0, s>>>(xp, h, w[0], w[1], w[2], w[3], n); break;
+    case 3: k_draft<T, 3><<<grid, 256, 0, s>>>(xp, h, w[0], w[1], w[2], w[3], n); break;
+    case 4: k_draft<T, 4><<<grid, 256, 0, s>>>(xp, h, w[0], w[1], w[2], w[3], n); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return launched();
+}
+
+cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int nt, long long n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  return dt == F32 ? draft_t<float>(x, h, w, nt, n, s) : draft_t<bf16>(x, h, w, nt, n, s);
+}
+
+// ---------------------------------------------------------------------------
+// Paid check + forward (Eqs. 3-5), fused so h_f is read once: each thread
+// rebuilds h_d from u and the history exactly as k_draft does, accumulates
+// |h_d - h_f|, |h_f|, (h_d - h_f)^2, h_f^2, and (Verify arm) stores h_d over
+// u.  Reduction: warp shuffles, then shared memory, then the 8 CTAs of a
+// thread-block cluster combine through distributed shared memory; one
+// partial per cluster goes to the workspace and a one-block kernel adds the
+// partials in a fixed order (deterministic run to run).
+// ---------------------------------------------------------------------------
+constexpr int VERIFY_THREADS = 256;
+constexpr int VERIFY_CLUSTER = 8;
+
+static int verify_grid(long long n) {
+  long long nvec = n / 4 + 1;
+  long long want = (nvec + VERIFY_THREADS - 1) / VERIFY_THREADS;
+  long long cap = (long long)num_sms() * 4;
+  if (want > cap) want = cap;
+  want = (want + VERIFY_CLUSTER - 1) / VERIFY_CLUSTER * VERIFY_CLUSTER;
+  if (want < VERIFY_CLUSTER) want = VERIFY_CLUSTER;
+  return (int)want;
+}
+
+size_t verify_workspace_bytes(long long n) {
+  return (size_t)(verify_grid(n) / VERIFY_CLUSTER) * 4 * sizeof(double);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+template <class T, int NT>
+__global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_THREADS)
+    k_verify(T* __restrict__ u, Hist4 h, float w0, float w1, float w2, float w3, const T* __restrict__ hf,
+             long long n, int write_draft, double* __restrict__ partials) {
+  constexpr int V = VecN<T>::n;
+  const float w[4] = {w0, w1, w2, w3};
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+  const long long nvec = n / V;
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += stride) {
+    float a[V], f[V];
+    draft_vec<T, NT>(u, h, w, i, a);
+    ld16(hf + i * V, f);
+#pragma unroll
+    for (int q = 0; q < V; ++q) {
+      const float ad = round_to(a[q], (T*)nullptr);  // h_d as it would be forwarded
+      const float d = ad - f[q];
+      s0 += fabsf(d);
+      s1 += fabsf(f[q]);
+      s2 += d * d;
+      s3 += f[q] * f[q];
+    }
+    if (write_draft) st16(u + i * V, a);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < n - nvec * V) {
+    const long long i = nvec * V + threadIdx.x;
+    const float a = round_to(draft_scalar<T, NT>(u, h, w, i), (T*)nullptr);
+    const float f = to_f(hf[i]);
+    const float d = a - f;
+    s0 += fabsf(d); s1 += fabsf(f); s2 += d * d; s3 += f * f;
+    if (write_draft) u[i] = from_f<T>(a);
+  }
+  s0 = warp_sum(s0); s1 = warp_sum(s1); s2 = warp_sum(s2); s3 = warp_sum(s3);
+  __shared__ float wsum[VERIFY_THREADS / 32][4];
+  __shared__ double bsum[4];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) { wsum[warp][0] = s0; wsum[warp][1] = s1; wsum[warp][2] = s2; wsum[warp][3] = s3; }
+  __syncthreads();
+  if (threadIdx.x < 4) {
+    double t = 0.0;
+    for (int k = 0; k < VERIFY_THREADS / 32; ++k) t += (double)wsum[k][threadIdx.x];
+    bsum[threadIdx.x] = t;
+  }
+  cg::cluster_group cluster = cg::this_cluster();
+  cluster.sync();
+  if (cluster.block_rank() == 0 && threadIdx.x < 4) {
+    double t = 0.0;
+    for (unsigned r = 0; r < cluster.num_blocks(); ++r) {
+      const double* rb = cluster.map_shared_rank(bsum, r);
+      t += rb[threadIdx.x];
+    }
+    partials[(size_t)(blockIdx.x / VERIFY_CLUSTER) * 4 + threadIdx.x] = t;
+  }
+  cluster.sync();
+}
+
+__global__ void k_verify_finish(const double* __restrict__ partials, int nparts, double* __restrict__ sums) {
+  if (threadIdx.x < 4) {
+    double t = 0.0;
+    for (int k = 0; k < nparts; ++k) t += partials[(size_t)k * 4 + threadIdx.x];
+    sums[threadIdx.x] = t;
+  }
+}
+
+template <class T>
+static cudaError_t verify_t(void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
+                           int write_draft, double* sums, void* ws, cudaStream_t s) {
+  const int grid = verify_grid(n);
+  double* parts = reinterpret_cast<double*>(ws);
+  T* up = reinterpret_cast<T*>(u);
+  const T* fp = reinterpret_cast<const T*>(hf);
+  switch (nt) {
+    case 1: k_verify<T, 1><<<grid, VERIFY_THREADS, 0, s>>>(up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    case 2: k_verify<T, 2><<<grid, VERIFY_THREADS, 0, s>>>(up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    case 3: k_verify<T, 3><<<grid, VERIFY_THREADS, 0, s>>>(up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    case 4: k_verify<T, 4><<<grid, VERIFY_THREADS, 0, s>>>(up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    default: return cudaErrorInvalidValue;
+  }
+  cudaError_t e = launched();
+  if (e != cudaSuccess) return e;
+  k_verify_finish<<<1, 32, 0, s>>>(parts, grid / VERIFY_CLUSTER, sums);
+  return launched();
+}
+
+cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
+                          int write_draft, double* sums, void* ws, cudaStream_t s) {
+  if (n <= 0) return cudaErrorInvalidValue;
+  return dt == F32 ? verify_t<float>(u, h, w, nt, hf, n, write_draft, sums, ws, s)
+                   : verify_t<bf16>(u, h, w, nt, hf, n, write_draft, sums, ws, s);
+}
+
+// ---------------------------------------------------------------------------
+// adaLN branch input: LN(x) (no affine, eps 1e-6) * (1 + scale_b) + shift_b.
+// One warp per row; the row is read three times (mean, variance, output),
+// the re-reads hit L1.
+// ---------------------------------------------------------------------------
+template <class T>
+__global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
+                                                const float* __restrict__ shift, const float* __restrict__ scale,
+                                                int mod_stride, int seg_split, int rpb0, int rpb1) {
+  constexpr int V = VecN<T>::n;
+  const long long r = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const T* xr = x + r * C;
+  const int nv = C / V;
+  float s = 0.f;
+  for (int k = lane; k < nv; k += 32) {
+    float a[V];
+    ld16(xr + k * V, a);
+#pragma unroll
+    for (int q = 0; q < V; ++q) s += a[q];
+  }
+  s = warp_sum(s);
+  const float mean = s / C;
+  float ss = 0.f;
+  for (int k = lane; k < nv; k += 32) {
+    float a[V];
+    ld16(xr + k * V, a);
+#pragma unroll
+    for (int q = 0; q < V; ++q) { const float d = a[q] - mean; ss += d * d; }
+  }
+  ss = warp_sum(ss);
+  const float rstd = rsqrtf(ss / C + 1e-6f);
+  const int b = (int)(r < seg_split ? r / rpb0 : (r - seg_split) / rpb1);
+  const float* sh = shift + (size_t)b * mod_stride;
+  const float* sc = scale + (size_t)b * mod_stride;
+  T* orow = out + r * C;
+  for (int k = lane; k < nv; k += 32) {
+    float a[V];
+    ld16(xr + k * V, a);
+#pragma unroll
+    for (int q = 0; q < V; ++q) {
+      const int c = k * V + q;
+      a[q] = (a[q] - mean) * rstd * (1.0f + sc[c]) + sh[c];
+    }
+    st16(orow + k * V, a);
+  }
+}
+
+cudaError_t launch_ln_mod(DType dt, const void* x, void* out, long long rows, int C, const float* shift,
+                          const float* scale, int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  const unsigned grid = (unsigned)((rows + 7) / 8);
+  if (dt == F32)
+    k_ln_mod<float><<<grid, 256, 0, s>>>((const float*)x, (float*)out, rows, C, shift, scale, mod_stride, seg_split,
+                                         rpb0, rpb1);
+  else
+    k_ln_mod<bf16><<<grid, 256, 0, s>>>((const bf16*)x, (bf16*)out, rows, C, shift, scale, mod_stride, seg_split,
+                                        rpb0, rpb1);
+  return launched();
+}
+
+// ---------------------------------------------------------------------------
+// Conditioning GEMV for a handful of rows: y[b, n] = f(sum_k W[n,k] g(x[b,k]) + bias[n]).
+// x sits in shared memory; each warp produces 4 outputs at a time so one
+// shared-memory read of x feeds 4 weight rows.
+// ---------------------------------------------------------------------------
+constexpr int LS_WARPS = 8;
+constexpr int LS_NPW = 4;
+
+template <class TW, int BMAX>
+__global__ void __launch_bounds__(LS_WARPS * 32) k_linear_small(const float* __restrict__ x, int B, int K,
+                                                                const TW* __restrict__ W, const TW* __restrict__ bias,
+                                                                int N, float* __restrict__ y, int ldy, int silu_in,
+                                                                int silu_out) {
+  extern __shared__ float xs[];
+  for (int i = threadIdx.x; i < B * K; i += blockDim.x) {
+    const float v = x[i];
+    xs[i] = silu_in ? silu(v) : v;
+  }
+  __syncthreads();
+  constexpr int V = VecN<TW>::n;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nv = K / V;
+  for (int n0 = (blockIdx.x * LS_WARPS + warp) * LS_NPW; n0 < N; n0 += gridDim.x * LS_WARPS * LS_NPW) {
+    float acc[LS_NPW][BMAX];
+#pragma unroll
+    for (int a = 0; a < LS_NPW; ++a)
+#pragma unroll
+      for (int b = 0; b < BMAX; ++b) acc[a][b] = 0.f;
+    for (int k = lane; k < nv; k += 32) {
+      float wv[LS_NPW][V];
+#pragma unroll
+      for (int a = 0; a < LS_NPW; ++a) {
+        if (n0 + a < N) ld16(W + (size_t)(n0 + a) * K + k * V, wv[a]);
+        else {
+#pragma unroll
+          for (int q = 0; q < V; ++q) wv[a][q] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int b = 0; b < BMAX; ++b) {
+        if (b < B) {
+          const float* xb = xs + b * K + k * V;
+#pragma unroll
+          for (int q = 0; q < V; ++q) {
+            const float xv = xb[q];
+#pragma unroll
+            for (int a = 0; a < LS_NPW; ++a) acc[a][b] = fmaf(wv[a][q], xv, acc[a][b]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int a = 0; a < LS_NPW; ++a) {
+#pragma unroll
+      for (int b = 0; b < BMAX; ++b) {
+        if (b < B) {
+          const float t = warp_sum(acc[a][b]);
+          if (lane == 0 && n0 + a < N) {
+            float v = t + (bias ? to_f(bias[n0 + a]) : 0.f);
+            y[(size_t)b * ldy + n0 + a] = silu_out ? silu(v) : v;
+          }
+        }
+      }
+    }
+  }
+}
+
+template <class TW, int BMAX>
+static cudaError_t linear_small_t(const float* x, int B, int K, const void* W, const void* bias, int N, float* y,
+                                  int ldy, int silu_in, int silu_out, cudaStream_t s) {
+  const size_t smem = (size_t)B * K * sizeof(float);
+  auto fn = k_linear_small<TW, BMAX>;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  int blocks = (N + LS_WARPS * LS_NPW - 1) / (LS_WARPS * LS_NPW);
+  if (blocks > num_sms() * 2) blocks = num_sms() * 2;
+  fn<<<blocks, LS_WARPS * 32, smem, s>>>(x, B, K, (const TW*)W, (const TW*)bias, N, y, ldy, silu_in, silu_out);
+  return launched();
+}
+
+cudaError_t launch_linear_small(DType wt, const float* x, int B, int K, const void* W, const void* bias, int N,
+                                float* y, int ldy, int silu_in, int silu_out, cudaStream_t s) {
+  if ((size_t)B * K * sizeof(float) > 200 * 1024) return cudaErrorInvalidValue;
+  if (wt == F32) {
+    if (K % 4) return cudaErrorInvalidValue;
+    if (B <= 2) return linear_small_t<float, 2>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
+    if (B <= 8) return linear_small_t<float, 8>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
+    if (B <= 16) return linear_small_t<float, 16>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
+    if (B <= 32) return linear_small_t<float, 32>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
+  } else {
+    if (K % 8) return cudaErrorInvalidValue;
+    if (B <= 2) return linear_small_t<bf16, 2>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
+    if (B <= 8) return linear_small_t<bf16, 8>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
+    if (B <= 16) return linear_small_t<bf16, 16>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
+    if (B <= 32) return linear_small_t<bf16, 32>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+// Sinusoidal timestep features: [cos(t f_k) | sin(t f_k)], f_k = 10000^(-k/half).
+__global__ void k_sinusoid(float t, float* out, int dim) {
+  const int half = dim / 2;
+  for (int k = threadIdx.x; k < half; k += blockDim.x) {
+    const double f = exp(-log(10000.0) * (double)k / (double)half);
+    const double a = (double)t * f;
+    out[k] = (float)cos(a);
+    out[k + half] = (float)sin(a);
+  }
+}
+
+cudaError_t launch_sinusoid(float t, float* out, int dim, cudaStream_t s) {
+  k_sinusoid<<<1, 128, 0, s>>>(t, out, dim);
+  return launched();
+}
+
+// c[b] = e (+ y_emb[label_b]); csilu = SiLU(c).
+template <class TW>
+__global__ void k_cond_finish(const float* __restrict__ e, const TW* __restrict__ y_emb, const int* __restrict__ labels,
+                              int B, int C, float* __restrict__ c_out, float* __restrict__ csilu) {
+  const int b = blockIdx.x;
+  for (int k = threadIdx.x; k < C; k += blockDim.x) {
+    float v = e[k];
+    if (y_emb) v += to_f(y_emb[(size_t)labels[b] * C + k]);
+    c_out[(size_t)b * C + k] = v;
+    csilu[(size_t)b * C + k] = silu(v);
+  }
+}
+
+cudaError_t launch_cond_finish(DType wt, const float* e, const void* y_emb, const int* labels, int B, int C,
+                               float* c_out, float* csilu_out, cudaStream_t s) {
+  if (wt == F32)
+    k_cond_finish<float><<<B, 256, 0, s>>>(e, (const float*)y_emb, labels, B, C, c_out, csilu_out);
+  else
+    k_cond_finish<bf16><<<B, 256, 0, s>>>(e, (const bf16*)y_emb, labels, B, C, c_out, csilu_out);
+  return launched();
+}
+
+// Patch features of the model batch (latent sample b % B_lat): row
+// b*N_img + token, feature (channel, frame offset, row offset, col offset).
+template <class T>
+__global__ void k_patchify(const float* __restrict__ lat, int B_lat, int B_model, int Cin, int F, int H, int W, int p,
+                           int pt, T* __restrict__ out) {
+  const int Ff = F > 0 ? F : 1, ptt = F > 0 ? pt : 1;
+  const int gf = Ff / ptt, gh = H / p, gw = W / p;
+  const int P = ptt * p * p, feat = Cin * P;
+  const long long total = (long long)B_model * gf * gh * gw * feat;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+    const int f = (int)(i % feat);
+    const long long row = i / feat;
+    const int tok = (int)(row % ((long long)gf * gh * gw));
+    const int b = (int)(row / ((long long)gf * gh * gw));
+    const int c = f / P, o = f % P;
+    const int ot = o / (p * p), oh = (o / p) % p, ow = o % p;
+    const int tw = tok % gw, th = (tok / gw) % gh, tf = tok / (gw * gh);
+    const int zf = tf * ptt + ot, zh = th * p + oh, zw = tw * p + ow;
+    const long long src = ((((long long)(b % B_lat) * Cin + c) * Ff + zf) * H + zh) * W + zw;
+    out[i] = from_f<T>(lat[src]);
+  }
+}
+
+cudaError_t launch_patchify(DType dt, const float* latent, int B_lat, int B_model, int Cin, int F, int H, int W,
+                            int p, int pt, void* out, cudaStream_t s) {
+  const int grid = num_sms() * 4;
+  if (dt == F32) k_patchify<float><<<grid, 256, 0, s>>>(latent, B_lat, B_model, Cin, F, H, W, p, pt, (float*)out);
+  else k_patchify<bf16><<<grid, 256, 0, s>>>(latent, B_lat, B_model, Cin, F, H, W, p, pt, (bf16*)out);
+  return launched();
+}
+
+template <class T>
+__global__ void k_convert(const float* __restrict__ in, T* __restrict__ out, long long n) {
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
+    out[i] = from_f<T>(in[i]);
+}
+
+cudaError_t launch_convert(DType dt, const float* in, void* out, long long n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int grid = num_sms() * 4;
+  if (dt == F32) k_convert<float><<<grid, 256, 0, s>>>(in, (float*)out, n);
+  else k_convert<bf16><<<grid, 256, 0, s>>>(in, (bf16*)out, n);
+  return launched();
+}
+
+// Guidance + sampler update of the latent: g = out_u + s (out_c - out_u)
+// (or out), x <- c1 x + c2 g, reading the model output through the
+// unpatchify index map.  Euler: c1 = 1, c2 = sigma_{i+1} - sigma_i.  DDIM:
+// c1 = sqrt(a_prev / a_t), c2 = sqrt(1 - a_prev) - sqrt(a_prev (1 - a_t) / a_t).
+__global__ void k_sampler(const float* __restrict__ mo, float* __restrict__ lat, int B_lat, int cfg, float cfg_scale,
+                          int Cin, int Cout, int F, int H, int W, int p, int pt, float c1, float c2) {
+  const int Ff = F > 0 ? F : 1, ptt = F > 0 ? pt : 1;
+  const int gh = H / p, gw = W / p, gf = Ff / ptt;
+  const int P = ptt * p * p;
+  const long long ntok = (long long)gf * gh * gw;
+  const long long total = (long long)B_lat * Cin * Ff * H * W;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+    const int zw = (int)(i % W);
+    const int zh = (int)((i / W) % H);
+    const int zf = (int)((i / ((long long)W * H)) % Ff);
+    const int c = (int)((i / ((long long)W * H * Ff)) % Cin);
+    const int b = (int)(i / ((long long)W * H * Ff * Cin));
+    const long long tok = ((long long)(zf / ptt) * gh + zh / p) * gw + zw / p;
+    const int f = c * P + ((zf % ptt) * p + zh % p) * p + zw % p;
+    const long long fo = (long long)Cout * P;
+    float g = mo[((long long)b * ntok + tok) * fo + f];
+    if (cfg) {
+      const float gu = mo[((long long)(b + B_lat) * ntok + tok) * fo + f];
+      g = gu + cfg_scale * (g - gu);
+    }
+    lat[i] = c1 * lat[i] + c2 * g;
+  }
+}
+
+cudaError_t launch_sampler(const float* model_out, float* latent, int B_lat, int cfg, float cfg_scale, int Cin,
+                           int Cout, int F, int H, int W, int p, int pt, float c1, float c2, cudaStream_t s) {
+  k_sampler<<<num_sms() * 2, 256, 0, s>>>(model_out, latent, B_lat, cfg, cfg_scale, Cin, Cout, F, H, W, p, pt, c1, c2);
+  return launched();
+}
+
+// Seeded N(0,1) latent: SplitMix64 word k = mix(seed + (k+1) * golden),
+// u = ((w >> 11) + 0.5) 2^-53, Box-Muller on word pairs (2m, 2m+1).
+__device__ __forceinline__ unsigned long long splitmix_word(unsigned long long seed, unsigned long long k) {
+  unsigned long long z = seed + (k + 1ull) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__global__ void k_noise(unsigned long long seed, float* __restrict__ out, long long n) {
+  const long long pairs = (n + 1) / 2;
+  for (long long m = (long long)blockIdx.x * blockDim.x + threadIdx.x; m < pairs; m += (long long)gridDim.x * blockDim.x) {
+    const double u1 = ((double)(splitmix_word(seed, 2 * m) >> 11) + 0.5) * 0x1.0p-53;
+    const double u2 = ((double)(splitmix_word(seed, 2 * m + 1) >> 11) + 0.5) * 0x1.0p-53;
+    const double r = sqrt(-2.0 * log(u1));
+    double sn, cs;
+    sincos(2.0 * 3.141592653589793 * u2, &sn, &cs);
+    out[2 * m] = (float)(r * cs);
+    if (2 * m + 1 < n) out[2 * m + 1] = (float)(r * sn);
+  }
+}
+
+cudaError_t launch_noise(unsigned long long seed, float* out, long long n, cudaStream_t s) {
+  k_noise<<<num_sms() * 2, 256, 0, s>>>(seed, out, n);
+  return launched();
+}
+
+// Fixed 2-D sin-cos position embedding replicated over B samples:
+// channels [0, C/2) encode the patch row, [C/2, C) the column, each half
+// [sin(pos w_k) | cos(pos w_k)], w_k = 10000^(-k/(C/4)).
+template <class T>
+__global__ void k_pos2d(T* __restrict__ out, int B, int gh, int gw, int C) {
+  const int q = C / 4;
+  const long long total = (long long)B * gh * gw * C;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
+    const int c = (int)(i % C);
+    const int tok = (int)((i / C) % ((long long)gh * gw));
+    const int half = c / (C / 2), cc = c % (C / 2);
+    const double pos = half == 0 ? (double)(tok / gw) : (double)(tok % gw);
+    const int k = cc % q;
+    const double a = pos * pow(10000.0, -(double)k / (double)q);
+    out[i] = from_f<T>((float)(cc < q ? sin(a) : cos(a)));
+  }
+}
+
+cudaError_t launch_pos2d(DType dt, void* out, int B, int gh, int gw, int C, cudaStream_t s) {
+  const int grid = num_sms() * 4;
+  if (dt == F32) k_pos2d<float><<<grid, 256, 0, s>>>((float*)out, B, gh, gw, C);
+  else k_pos2d<bf16><<<grid, 256, 0, s>>>((bf16*)out, B, gh, gw, C);
+  return launched();
+}
+
+}  // namespace ff

@@ -1,0 +1,962 @@
+// Host runtime of the FeatFix cached denoising path and the C ABI of
+// include/featfix.h: context and workspace, the fixed schedule (Section 3.3),
+// the draft weights of Eq. 2, the per-step block loop (Eqs. 1-5), logs,
+// accounting, debug capture and kernel timing.
+#include "featfix.h"
+#include "featfix_ops.h"
+#include "ff_common.cuh"
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+using namespace ff;
+
+namespace {
+
+constexpr int NKCLASS = 5;
+
+struct Capture {
+  int step, layer;
+  void* in;
+  void* out;
+};
+
+struct TimedLaunch {
+  cudaEvent_t a, b;
+  double work;
+};
+
+}  // namespace
+
+struct featfix_ctx {
+  featfix_model_desc d;
+  DType dt;
+  int es;
+  int L, Bm, Nt, Ni, Ntot, C, H, hd, M, P, fin, fout;
+  long long T, E;
+  int gf, gh, gw;
+  std::vector<const void*> w;
+  cudaStream_t st;
+
+  void *xa = nullptr, *xb = nullptr, *xm = nullptr, *qkv = nullptr, *att = nullptr, *u1 = nullptr, *big = nullptr;
+  void *patches = nullptr, *pos = nullptr;
+  float *mod_a = nullptr, *mod_b = nullptr, *cvec = nullptr, *csilu = nullptr, *sinus = nullptr, *thid = nullptr,
+        *temb = nullptr, *mout = nullptr;
+  float2* rope = nullptr;
+  void* ring = nullptr;
+  int S = 0;
+  double* dsums = nullptr;
+  int max_logs = 0;
+  void* vws = nullptr;
+  size_t vws_bytes = 0;
+  float* h_latent = nullptr;  // device buffers of featfix_sample_host
+  void* h_cond = nullptr;
+
+  bool sched = false;
+  int steps = 0, K = 0, mode = 0;
+  unsigned flags = 0;
+  std::vector<unsigned char> kinds;
+  std::vector<int> keff;
+  std::vector<double> wts;
+  std::vector<char> isref;
+
+  int next_step = 0;
+  int head = 0, count = 0;
+  std::vector<std::pair<int, int>> log_sites;
+  featfix_counters cnt = {0, 0, 0, 0};
+  std::vector<Capture> caps;
+
+  bool timing[NKCLASS] = {false, false, false, false, false};
+  std::vector<TimedLaunch> pending[NKCLASS];
+  std::vector<cudaEvent_t> evpool;
+  double tms[NKCLASS] = {0, 0, 0, 0, 0};
+  double twork[NKCLASS] = {0, 0, 0, 0, 0};
+  long long tcount[NKCLASS] = {0, 0, 0, 0, 0};
+
+  std::string err;
+};
+
+namespace {
+
+featfix_status fail(featfix_ctx* c, featfix_status s, const std::string& msg) {
+  if (c) c->err = msg;
+  return s;
+}
+
+#define FF_CK(call)                                                                                \
+  do {                                                                                             \
+    cudaError_t e__ = (call);                                                                      \
+    if (e__ != cudaSuccess)                                                                        \
+      return fail(ctx, FEATFIX_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e__));     \
+  } while (0)
+
+int n_layers(const featfix_model_desc& d) { return d.arch == FEATFIX_ARCH_MMDIT ? d.n_dual + d.n_single : d.n_dual; }
+
+int patch_vol(const featfix_model_desc& d) { return (d.lat_f > 0 ? d.patch_t : 1) * d.patch * d.patch; }
+
+int img_tokens(const featfix_model_desc& d) {
+  const int gf = d.lat_f > 0 ? d.lat_f / d.patch_t : 1;
+  return gf * (d.lat_h / d.patch) * (d.lat_w / d.patch);
+}
+
+std::string check_desc(const featfix_model_desc* d) {
+  if (!d) return "null model description";
+  if (d->arch != FEATFIX_ARCH_DIT && d->arch != FEATFIX_ARCH_MMDIT) return "unknown arch";
+  if (d->n_dual < 0 || d->n_single < 0 || n_layers(*d) < 1) return "no blocks";
+  if (d->arch == FEATFIX_ARCH_DIT && (d->n_single != 0 || d->txt_tokens != 0)) return "DiT has no single blocks or text";
+  if (d->hidden <= 0 || d->heads <= 0 || d->head_dim <= 0 || d->hidden != d->heads * d->head_dim)
+    return "hidden != heads * head_dim";
+  if (d->head_dim % 8 || d->head_dim > 128) return "head_dim must be a multiple of 8, <= 128";
+  if (d->hidden % 32 || d->mlp <= 0 || d->mlp % 32) return "hidden and mlp must be multiples of 32";
+  if (d->in_ch <= 0 || d->out_ch < d->in_ch) return "bad channel counts";
+  if (d->patch <= 0 || d->lat_h % d->patch || d->lat_w % d->patch || d->lat_h <= 0 || d->lat_w <= 0)
+    return "latent not divisible by patch";
+  if (d->lat_f < 0 || (d->lat_f > 0 && (d->patch_t <= 0 || d->lat_f % d->patch_t))) return "bad temporal patch";
+  if (d->txt_tokens < 0) return "bad text length";
+  if (d->batch <= 0) return "bad batch";
+  const int bm = d->batch * (d->cfg ? 2 : 1);
+  if (bm > 32) return "model batch above 32";
+  if (d->arch == FEATFIX_ARCH_DIT && d->n_classes <= 0) return "DiT needs classes";
+  if (d->rope_dims != 0 && d->rope_dims != 2 && d->rope_dims != 3) return "rope_dims must be 0, 2 or 3";
+  if (d->rope_dims == 3 && d->lat_f <= 0) return "3-D rotary needs frames";
+  if (d->rope_dims != 0 && d->arch != FEATFIX_ARCH_MMDIT) return "rotary positions are for MMDiT";
+  if (d->dtype != FEATFIX_DTYPE_F32 && d->dtype != FEATFIX_DTYPE_BF16) return "bad dtype";
+  if (d->sampler != FEATFIX_SAMPLER_EULER && d->sampler != FEATFIX_SAMPLER_DDIM) return "bad sampler";
+  if (d->arch == FEATFIX_ARCH_DIT && d->hidden % 4) return "position embedding needs hidden % 4 == 0";
+  const int fo = patch_vol(*d) * d->out_ch, fi = patch_vol(*d) * d->in_ch;
+  const int v = d->dtype == FEATFIX_DTYPE_F32 ? 4 : 8;
+  if (fo % v || fi % v) return "patch feature widths must be multiples of the 16-byte vector";
+  return "";
+}
+
+// ---------------------------------------------------------------------------
+// schedule and draft weights
+// ---------------------------------------------------------------------------
+// Weights w_j of the j-th newest refresh increment so that the draft's
+// forecast is sum_j w_j R_{s_j}.
+//  default: Lagrange basis of the polynomial through the nodes, evaluated at
+//           t -- equal to the Taylor series of Eq. 2 whose derivatives are
+//           those of that polynomial at s_0.
+//  recursive: Delta^(0)_j = R_j, Delta^(k)_j = (Delta^(k-1)_j -
+//           Delta^(k-1)_{j+1}) / (s_j - s_{j+1}), forecast
+//           sum_k (t - s_0)^k / k! Delta^(k)_0, expanded over the R_j.
+void draft_weights(const std::vector<int>& s, int t, bool recursive, double* w) {
+  const int n = (int)s.size();
+  for (int j = 0; j < 4; ++j) w[j] = 0.0;
+  if (!recursive) {
+    for (int j = 0; j < n; ++j) {
+      double p = 1.0;
+      for (int m = 0; m < n; ++m)
+        if (m != j) p *= (double)(t - s[m]) / (double)(s[j] - s[m]);
+      w[j] = p;
+    }
+    return;
+  }
+  // lvl[j][r]: coefficient of R_r in Delta^(k)_j
+  std::vector<std::vector<double>> lvl(n, std::vector<double>(n, 0.0));
+  for (int j = 0; j < n; ++j) lvl[j][j] = 1.0;
+  double fact = 1.0, pw = 1.0;
+  for (int r = 0; r < n; ++r) w[r] += lvl[0][r];
+  for (int k = 1; k < n; ++k) {
+    std::vector<std::vector<double>> nx(n - k, std::vector<double>(n, 0.0));
+    for (int j = 0; j < n - k; ++j)
+      for (int r = 0; r < n; ++r) nx[j][r] = (lvl[j][r] - lvl[j + 1][r]) / (double)(s[j] - s[j + 1]);
+    lvl.swap(nx);
+    fact *= k;
+    pw *= (double)(t - s[0]);
+    for (int r = 0; r < n; ++r) w[r] += pw / fact * lvl[0][r];
+  }
+}
+
+featfix_status plan_core(int steps, int L, const int* refresh, int n_refresh, int K, const featfix_site* sites,
+                         int n_sites, int mode, unsigned flags, std::vector<unsigned char>& kinds,
+                         std::vector<int>& keff, std::vector<double>& wts, std::vector<char>& isref,
+                         std::string& err) {
+  if (mode < FEATFIX_MODE_FEATFIX || mode > FEATFIX_MODE_VANILLA) { err = "unknown mode"; return FEATFIX_ERR_INVALID_ARG; }
+  if (steps < 1 || L < 1) { err = "steps and layers must be positive"; return FEATFIX_ERR_SCHEDULE; }
+  if (K < 0 || K > 3) { err = "draft order must be in [0, 3]"; return FEATFIX_ERR_SCHEDULE; }
+  if (n_refresh < 1 || !refresh) { err = "no refresh steps"; return FEATFIX_ERR_SCHEDULE; }
+  if (n_sites < 0 || (n_sites > 0 && !sites)) { err = "bad site list"; return FEATFIX_ERR_INVALID_ARG; }
+  isref.assign(steps, 0);
+  for (int k = 0; k < n_refresh; ++k) {
+    const int r = refresh[k];
+    if (r < 0 || r >= steps) { err = "refresh step out of range"; return FEATFIX_ERR_SCHEDULE; }
+    if (isref[r]) { err = "duplicate refresh step"; return FEATFIX_ERR_SCHEDULE; }
+    isref[r] = 1;
+  }
+  if (!isref[0]) { err = "step 0 must be a full refresh"; return FEATFIX_ERR_SCHEDULE; }
+  std::vector<char> issite((size_t)steps * L, 0);
+  for (int k = 0; k < n_sites; ++k) {
+    const int i = sites[k].step, l = sites[k].layer;
+    if (i < 0 || i >= steps || l < 0 || l >= L) { err = "site out of range"; return FEATFIX_ERR_SCHEDULE; }
+    if (isref[i]) { err = "site on a refresh step"; return FEATFIX_ERR_SCHEDULE; }
+    if (issite[(size_t)i * L + l]) { err = "duplicate site"; return FEATFIX_ERR_SCHEDULE; }
+    issite[(size_t)i * L + l] = 1;
+  }
+  kinds.assign((size_t)steps * L, FEATFIX_PLAN_DRAFT);
+  keff.assign(steps, -1);
+  wts.assign((size_t)steps * 4, 0.0);
+  std::vector<int> nodes;  // refresh steps, newest first
+  for (int i = 0; i < steps; ++i) {
+    if (isref[i]) {
+      nodes.insert(nodes.begin(), i);
+      if ((int)nodes.size() > K + 1) nodes.resize(K + 1);
+    }
+    const bool all_exact = mode == FEATFIX_MODE_VANILLA || isref[i];
+    for (int l = 0; l < L; ++l) {
+      unsigned char k = FEATFIX_PLAN_DRAFT;
+      if (all_exact) k = FEATFIX_PLAN_EXACT;
+      else if (issite[(size_t)i * L + l]) k = FEATFIX_PLAN_SITE;
+      kinds[(size_t)i * L + l] = k;
+    }
+    if (!all_exact) {
+      const int ke = std::min(K, (int)nodes.size() - 1);
+      keff[i] = ke;
+      std::vector<int> s(nodes.begin(), nodes.begin() + ke + 1);
+      draft_weights(s, i, (flags & FEATFIX_FLAG_TAYLOR_RECURSIVE) != 0, &wts[(size_t)i * 4]);
+    }
+  }
+  return FEATFIX_OK;
+}
+
+// ---------------------------------------------------------------------------
+// samplers (host constants)
+// ---------------------------------------------------------------------------
+double ddim_alpha_bar(int tau) {
+  double ab = 1.0;
+  for (int k = 0; k <= tau; ++k) ab *= 1.0 - (1e-4 + (0.02 - 1e-4) * (double)k / 999.0);
+  return ab;
+}
+
+double model_time(const featfix_ctx* c, int i) {
+  if (c->d.sampler == FEATFIX_SAMPLER_EULER) return 1000.0 * (1.0 - (double)i / c->steps);
+  return (double)(1000 - (1000 / c->steps) * (i + 1));
+}
+
+void sampler_coeffs(const featfix_ctx* c, int i, float* c1, float* c2) {
+  if (c->d.sampler == FEATFIX_SAMPLER_EULER) {
+    *c1 = 1.0f;
+    *c2 = (float)((1.0 - (double)(i + 1) / c->steps) - (1.0 - (double)i / c->steps));
+    return;
+  }
+  const int stride = 1000 / c->steps;
+  const double at = ddim_alpha_bar(1000 - stride * (i + 1));
+  const double ap = i + 1 < c->steps ? ddim_alpha_bar(1000 - stride * (i + 2)) : 1.0;
+  *c1 = (float)std::sqrt(ap / at);
+  *c2 = (float)(std::sqrt(1.0 - ap) - std::sqrt(ap * (1.0 - at) / at));
+}
+
+// ---------------------------------------------------------------------------
+// kernel timing
+// ---------------------------------------------------------------------------
+cudaEvent_t ev_get(featfix_ctx* c) {
+  if (!c->evpool.empty()) {
+    cudaEvent_t e = c->evpool.back();
+    c->evpool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+struct KTimer {
+  featfix_ctx* c;
+  int k;
+  double work;
+  cudaEvent_t a = nullptr;
+  KTimer(featfix_ctx* c_, int k_, double work_) : c(c_), k(k_), work(work_) {
+    if (c->timing[k]) {
+      a = ev_get(c);
+      cudaEventRecord(a, c->st);
+    }
+  }
+  ~KTimer() {
+    if (a) {
+      cudaEvent_t b = ev_get(c);
+      cudaEventRecord(b, c->st);
+      c->pending[k].push_back({a, b, work});
+    }
+  }
+};
+
+void timing_drain(featfix_ctx* c) {
+  for (int k = 0; k < NKCLASS; ++k) {
+    for (auto& t : c->pending[k]) {
+      float ms = 0.f;
+      if (cudaEventElapsedTime(&ms, t.a, t.b) == cudaSuccess) {
+        c->tms[k] += ms;
+        c->twork[k] += t.work;
+        c->tcount[k] += 1;
+      }
+      c->evpool.push_back(t.a);
+      c->evpool.push_back(t.b);
+    }
+    c->pending[k].clear();
+  }
+}
+
+// ---------------------------------------------------------------------------
+// building blocks
+// ---------------------------------------------------------------------------
+template <class T>
+T* at(void* base, long long elems, int es) {
+  return reinterpret_cast<T*>(reinterpret_cast<char*>(base) + elems * es);
+}
+void* off(void* base, long long elems, int es) { return reinterpret_cast<char*>(base) + elems * es; }
+const void* coff(const void* base, long long elems, int es) { return reinterpret_cast<const char*>(base) + elems * es; }
+
+cudaError_t dense(featfix_ctx* c, int M, int N, int K, const void* A, int lda, const void* W, const EpiArgs& e) {
+  KTimer tm(c, FEATFIX_KCLASS_GEMM, 2.0 * M * N * (double)K);
+  if (c->dt == BF16) return gemm_tc(M, N, K, A, lda, W, K, e, c->st);
+  return gemm_simt(c->dt, M, N, K, A, lda, W, K, e, c->st);
+}
+
+EpiArgs epi(void* out, int ldo, const void* bias) {
+  EpiArgs e = epi_plain(out, ldo);
+  e.bias = bias;
+  return e;
+}
+
+cudaError_t run_attention(featfix_ctx* c, const void* q, const void* k, const void* v, int ld, void* out, int ldo) {
+  const double N = c->Ntot;
+  KTimer tm(c, FEATFIX_KCLASS_ATTENTION, 4.0 * c->Bm * c->H * N * N * c->hd);
+  AttnArgs a;
+  a.q = q; a.k = k; a.v = v; a.ld_qkv = ld;
+  a.out = out; a.ld_out = ldo;
+  a.B = c->Bm; a.Nt = c->Nt; a.Ni = c->Ni; a.H = c->H; a.hd = c->hd;
+  return attention(c->dt, a, c->st);
+}
+
+cudaError_t modvec(featfix_ctx* c, int widx, int chunks, float* out) {
+  KTimer tm(c, FEATFIX_KCLASS_OTHER, 0);
+  return launch_linear_small(c->dt, c->csilu, c->Bm, c->C, c->w[widx], c->w[widx + 1], chunks * c->C, out,
+                             chunks * c->C, 0, 0, c->st);
+}
+
+cudaError_t ln_mod(featfix_ctx* c, const void* x, void* out, long long rows, const float* mod, int shift_chunk,
+                   int scale_chunk, int stride_chunks, int seg_split, int rpb0, int rpb1) {
+  KTimer tm(c, FEATFIX_KCLASS_OTHER, 0);
+  return launch_ln_mod(c->dt, x, out, rows, c->C, mod + shift_chunk * c->C, mod + scale_chunk * c->C,
+                       stride_chunks * c->C, seg_split, rpb0, rpb1, c->st);
+}
+
+// Exact DiT block B_l (Eq. 1): u -> out, optional history increment out - u.
+featfix_status block_dit(featfix_ctx* ctx, int l, const void* u, void* out, void* hist) {
+  const int C = ctx->C, M = ctx->M, es = ctx->es;
+  const long long T = ctx->T;
+  const int wb = 11 + 10 * l;
+  const auto& W = ctx->w;
+  FF_CK(modvec(ctx, wb, 6, ctx->mod_a));
+  FF_CK(ln_mod(ctx, u, ctx->xm, T, ctx->mod_a, 0, 1, 6, 0, 1, ctx->Ni));
+  FF_CK(dense(ctx, (int)T, 3 * C, C, ctx->xm, C, W[wb + 2], epi(ctx->qkv, 3 * C, W[wb + 3])));
+  FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, es), off(ctx->qkv, 2 * C, es), 3 * C, ctx->att, C));
+  EpiArgs e = epi(ctx->u1, C, W[wb + 5]);
+  e.gate = ctx->mod_a + 2 * C; e.gate_stride = 6 * C; e.rpb1 = ctx->Ni;
+  e.resid = u; e.ld_resid = C;
+  FF_CK(dense(ctx, (int)T, C, C, ctx->att, C, W[wb + 4], e));
+  FF_CK(ln_mod(ctx, ctx->u1, ctx->xm, T, ctx->mod_a, 3, 4, 6, 0, 1, ctx->Ni));
+  EpiArgs e1 = epi(ctx->big, M, W[wb + 7]);
+  e1.act = 1;
+  FF_CK(dense(ctx, (int)T, M, C, ctx->xm, C, W[wb + 6], e1));
+  EpiArgs e2 = epi(out, C, W[wb + 9]);
+  e2.gate = ctx->mod_a + 5 * C; e2.gate_stride = 6 * C; e2.rpb1 = ctx->Ni;
+  e2.resid = ctx->u1; e2.ld_resid = C;
+  if (hist) { e2.hist_base = u; e2.hist_out = hist; }
+  FF_CK(dense(ctx, (int)T, C, M, ctx->big, M, W[wb + 8], e2));
+  return FEATFIX_OK;
+}
+
+// Exact MMDiT two-stream block: per-stream modulation and projections,
+// joint attention.  Text rows [0, Bm*Nt), image rows after.
+featfix_status block_dual(featfix_ctx* ctx, int l, const void* u, void* out, void* hist) {
+  const int C = ctx->C, M = ctx->M, es = ctx->es;
+  const int wb = 10 + 20 * l;
+  const auto& W = ctx->w;
+  const long long rt = (long long)ctx->Bm * ctx->Nt, ri = (long long)ctx->Bm * ctx->Ni;
+  float* mi = ctx->mod_a;
+  float* mt = ctx->mod_b;
+  FF_CK(modvec(ctx, wb, 6, mi));
+  if (rt) FF_CK(modvec(ctx, wb + 2, 6, mt));
+  // stream s: 0 text, 1 image
+  for (int s = 0; s < 2; ++s) {
+    const long long r0 = s == 0 ? 0 : rt, rows = s == 0 ? rt : ri;
+    if (!rows) continue;
+    FF_CK(ln_mod(ctx, coff(u, r0 * C, es), off(ctx->xm, r0 * C, es), rows, s ? mi : mt, 0, 1, 6, 0, 1,
+                 s ? ctx->Ni : ctx->Nt));
+    const int wq = s ? wb + 4 : wb + 6;
+    EpiArgs e = epi(off(ctx->qkv, r0 * 3 * C, es), 3 * C, W[wq + 1]);
+    if (s == 1 && ctx->rope) {
+      e.rope = ctx->rope; e.rope_row0 = 0; e.rope_period = ctx->Ni; e.rope_cols = 2 * C; e.rope_hd = ctx->hd;
+    }
+    FF_CK(dense(ctx, (int)rows, 3 * C, C, off(ctx->xm, r0 * C, es), C, W[wq], e));
+  }
+  FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, es), off(ctx->qkv, 2 * C, es), 3 * C, ctx->att, C));
+  for (int s = 0; s < 2; ++s) {
+    const long long r0 = s == 0 ? 0 : rt, rows = s == 0 ? rt : ri;
+    if (!rows) continue;
+    float* m = s ? mi : mt;
+    const int rpb = s ? ctx->Ni : ctx->Nt;
+    const int wp = s ? wb + 8 : wb + 10;
+    EpiArgs e = epi(off(ctx->u1, r0 * C, es), C, W[wp + 1]);
+    e.gate = m + 2 * C; e.gate_stride = 6 * C; e.rpb1 = rpb;
+    e.resid = coff(u, r0 * C, es); e.ld_resid = C;
+    FF_CK(dense(ctx, (int)rows, C, C, off(ctx->att, r0 * C, es), C, W[wp], e));
+    FF_CK(ln_mod(ctx, off(ctx->u1, r0 * C, es), off(ctx->xm, r0 * C, es), rows, m, 3, 4, 6, 0, 1, rpb));
+    const int wf = s ? wb + 12 : wb + 16;
+    EpiArgs e1 = epi(off(ctx->big, r0 * M, es), M, W[wf + 1]);
+    e1.act = 1;
+    FF_CK(dense(ctx, (int)rows, M, C, off(ctx->xm, r0 * C, es), C, W[wf], e1));
+    EpiArgs e2 = epi(off(out, r0 * C, es), C, W[wf + 3]);
+    e2.gate = m + 5 * C; e2.gate_stride = 6 * C; e2.rpb1 = rpb;
+    e2.resid = off(ctx->u1, r0 * C, es); e2.ld_resid = C;
+    if (hist) { e2.hist_base = coff(u, r0 * C, es); e2.hist_out = off(hist, r0 * C, es); }
+    FF_CK(dense(ctx, (int)rows, C, M, off(ctx->big, r0 * M, es), M, W[wf + 2], e2));
+  }
+  return FEATFIX_OK;
+}
+
+// Exact MMDiT single-stream block: linear1 -> [q k v | GELU(mlp)] (the MLP
+// half written next to the attention output), joint attention, linear2.
+featfix_status block_single(featfix_ctx* ctx, int l, const void* u, void* out, void* hist) {
+  const int C = ctx->C, M = ctx->M;
+  const int j = l - ctx->d.n_dual;
+  const int wb = 10 + 20 * ctx->d.n_dual + 6 * j;
+  const auto& W = ctx->w;
+  const long long T = ctx->T, rt = (long long)ctx->Bm * ctx->Nt;
+  FF_CK(modvec(ctx, wb, 3, ctx->mod_a));
+  FF_CK(ln_mod(ctx, u, ctx->xm, T, ctx->mod_a, 0, 1, 3, (int)rt, ctx->Nt > 0 ? ctx->Nt : 1, ctx->Ni));
+  EpiArgs e = epi(ctx->qkv, 3 * C, W[wb + 3]);
+  e.split_col = 3 * C;
+  e.out2 = off(ctx->big, C, ctx->es);
+  e.ldo2 = C + M;
+  e.act = 1; e.act_col0 = 3 * C;
+  if (ctx->rope) {
+    e.rope = ctx->rope; e.rope_row0 = (int)rt; e.rope_period = ctx->Ni; e.rope_cols = 2 * C; e.rope_hd = ctx->hd;
+  }
+  FF_CK(dense(ctx, (int)T, 3 * C + M, C, ctx->xm, C, W[wb + 2], e));
+  FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, ctx->es), off(ctx->qkv, 2 * C, ctx->es), 3 * C, ctx->big,
+                      C + M));
+  EpiArgs e2 = epi(out, C, W[wb + 5]);
+  e2.gate = ctx->mod_a + 2 * C; e2.gate_stride = 3 * C;
+  e2.seg_split = (int)rt; e2.rpb0 = ctx->Nt > 0 ? ctx->Nt : 1; e2.rpb1 = ctx->Ni;
+  e2.resid = u; e2.ld_resid = C;
+  if (hist) { e2.hist_base = u; e2.hist_out = hist; }
+  FF_CK(dense(ctx, (int)T, C, C + M, ctx->big, C + M, W[wb + 4], e2));
+  return FEATFIX_OK;
+}
+
+featfix_status exact_block(featfix_ctx* ctx, int l, const void* u, void* out, void* hist) {
+  if (ctx->d.arch == FEATFIX_ARCH_DIT) return block_dit(ctx, l, u, out, hist);
+  if (l < ctx->d.n_dual) return block_dual(ctx, l, u, out, hist);
+  return block_single(ctx, l, u, out, hist);
+}
+
+// c = MLP(sinusoid(t)) (+ label embedding), SiLU(c) for the modulations.
+featfix_status conditioning(featfix_ctx* ctx, double t, const void* cond) {
+  KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+  const auto& W = ctx->w;
+  FF_CK(launch_sinusoid((float)t, ctx->sinus, 256, ctx->st));
+  FF_CK(launch_linear_small(ctx->dt, ctx->sinus, 1, 256, W[0], W[1], ctx->C, ctx->thid, ctx->C, 0, 1, ctx->st));
+  FF_CK(launch_linear_small(ctx->dt, ctx->thid, 1, ctx->C, W[2], W[3], ctx->C, ctx->temb, ctx->C, 0, 0, ctx->st));
+  const bool dit = ctx->d.arch == FEATFIX_ARCH_DIT;
+  FF_CK(launch_cond_finish(ctx->dt, ctx->temb, dit ? W[4] : nullptr, dit ? (const int*)cond : nullptr, ctx->Bm,
+                           ctx->C, ctx->cvec, ctx->csilu, ctx->st));
+  return FEATFIX_OK;
+}
+
+// Block-0 input: DiT patch embedding + position; MMDiT [text ; patches].
+featfix_status embed(featfix_ctx* ctx, const float* latent, const void* cond, void* x) {
+  const auto& d = ctx->d;
+  const int C = ctx->C, es = ctx->es;
+  const long long rt = (long long)ctx->Bm * ctx->Nt;
+  {
+    KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+    FF_CK(launch_patchify(ctx->dt, latent, d.batch, ctx->Bm, d.in_ch, d.lat_f, d.lat_h, d.lat_w, d.patch, d.patch_t,
+                          ctx->patches, ctx->st));
+  }
+  if (d.arch == FEATFIX_ARCH_DIT) {
+    EpiArgs e = epi(x, C, ctx->w[6]);
+    e.resid = ctx->pos; e.ld_resid = C;
+    FF_CK(dense(ctx, ctx->Bm * ctx->Ni, C, ctx->fin, ctx->patches, ctx->fin, ctx->w[5], e));
+  } else {
+    if (rt) {
+      KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+      FF_CK(launch_convert(ctx->dt, (const float*)cond, x, rt * C, ctx->st));
+    }
+    FF_CK(dense(ctx, ctx->Bm * ctx->Ni, C, ctx->fin, ctx->patches, ctx->fin, ctx->w[4], epi(off(x, rt * C, es), C, ctx->w[5])));
+  }
+  return FEATFIX_OK;
+}
+
+// Final layer on the image rows and the guided sampler update.
+featfix_status finish_step(featfix_ctx* ctx, int i, const void* x, float* latent) {
+  const auto& d = ctx->d;
+  const int C = ctx->C, es = ctx->es;
+  const bool dit = d.arch == FEATFIX_ARCH_DIT;
+  const int wm = dit ? 7 : 6;
+  const long long rt = (long long)ctx->Bm * ctx->Nt, ri = (long long)ctx->Bm * ctx->Ni;
+  FF_CK(modvec(ctx, wm, 2, ctx->mod_b));
+  FF_CK(ln_mod(ctx, coff(x, rt * C, es), ctx->xm, ri, ctx->mod_b, 0, 1, 2, 0, 1, ctx->Ni));
+  EpiArgs e = epi(ctx->mout, ctx->fout, ctx->w[wm + 3]);
+  e.out_f32 = 1;
+  FF_CK(dense(ctx, (int)ri, ctx->fout, C, ctx->xm, C, ctx->w[wm + 2], e));
+  float c1, c2;
+  sampler_coeffs(ctx, i, &c1, &c2);
+  KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+  FF_CK(launch_sampler(ctx->mout, latent, d.batch, d.cfg, d.cfg_scale, d.in_ch, d.out_ch, d.lat_f, d.lat_h, d.lat_w,
+                       d.patch, d.patch_t, c1, c2, ctx->st));
+  return FEATFIX_OK;
+}
+
+void* ring_slot(featfix_ctx* c, int l, int slot) {
+  return off(c->ring, ((long long)l * c->S + slot) * c->E, c->es);
+}
+
+Hist4 hist_ptrs(featfix_ctx* c, int l, int nt) {
+  Hist4 h = {{nullptr, nullptr, nullptr, nullptr}};
+  for (int j = 0; j < nt; ++j) h.p[j] = ring_slot(c, l, ((c->head - j) % c->S + c->S) % c->S);
+  return h;
+}
+
+void free_all(featfix_ctx* c) {
+  void* bufs[] = {c->xa, c->xb, c->xm, c->qkv, c->att, c->u1, c->big, c->patches, c->pos, c->mod_a, c->mod_b,
+                  c->cvec, c->csilu, c->sinus, c->thid, c->temb, c->mout, c->rope, c->ring, c->dsums, c->vws,
+                  c->h_latent, c->h_cond};
+  for (void* p : bufs)
+    if (p) cudaFree(p);
+  for (int k = 0; k < NKCLASS; ++k)
+    for (auto& t : c->pending[k]) { cudaEventDestroy(t.a); cudaEventDestroy(t.b); }
+  for (auto e : c->evpool) cudaEventDestroy(e);
+}
+
+featfix_status alloc(featfix_ctx* c, void** p, size_t bytes) {
+  if (cudaMalloc(p, bytes ? bytes : 16) != cudaSuccess) {
+    cudaGetLastError();
+    *p = nullptr;
+    return fail(c, FEATFIX_ERR_OOM, "device allocation of " + std::to_string(bytes) + " bytes failed");
+  }
+  return FEATFIX_OK;
+}
+
+// (cos, sin) of every image token / rotary pair: axis widths d/2,d/2 (2-D)
+// or d/8, 7d/16, 7d/16 (3-D); pair j of an axis of width w turns by
+// pos * 10000^(-2j/w).
+std::vector<float2> rope_table_host(const featfix_model_desc& d, int hd) {
+  std::vector<int> axes;
+  if (d.rope_dims == 2) axes = {hd / 2, hd / 2};
+  else {
+    const int t = hd / 8, hw = (hd - t) / 2;
+    axes = {t, hw, hd - t - hw};
+  }
+  const int gf = d.lat_f > 0 ? d.lat_f / d.patch_t : 1, gh = d.lat_h / d.patch, gw = d.lat_w / d.patch;
+  const int ni = gf * gh * gw;
+  std::vector<float2> tab((size_t)ni * (hd / 2));
+  for (int n = 0; n < ni; ++n) {
+    int pos[3];
+    if (d.rope_dims == 2) { pos[0] = (n / gw) % gh; pos[1] = n % gw; }
+    else { pos[0] = n / (gw * gh); pos[1] = (n / gw) % gh; pos[2] = n % gw; }
+    int col = 0;
+    for (size_t a = 0; a < axes.size(); ++a) {
+      for (int j = 0; j < axes[a] / 2; ++j, ++col) {
+        const double ang = pos[a] * std::pow(10000.0, -2.0 * j / axes[a]);
+        tab[(size_t)n * (hd / 2) + col] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+      }
+    }
+  }
+  return tab;
+}
+
+}  // namespace
+
+// ============================================================================
+// C ABI
+// ============================================================================
+extern "C" {
+
+const char* featfix_status_string(featfix_status s) {
+  switch (s) {
+    case FEATFIX_OK: return "ok";
+    case FEATFIX_ERR_INVALID_ARG: return "invalid argument";
+    case FEATFIX_ERR_SCHEDULE: return "schedule rule violated";
+    case FEATFIX_ERR_STATE: return "call out of order";
+    case FEATFIX_ERR_OOM: return "out of device memory";
+    case FEATFIX_ERR_CUDA: return "CUDA error";
+    case FEATFIX_ERR_UNSUPPORTED: return "unsupported";
+  }
+  return "unknown status";
+}
+
+long long featfix_launch_count(void) { return launches_total(); }
+
+const char* featfix_last_error(const featfix_ctx* ctx) { return ctx ? ctx->err.c_str() : "null context"; }
+
+int featfix_weight_count(const featfix_model_desc* d) {
+  if (!check_desc(d).empty()) return -1;
+  if (d->arch == FEATFIX_ARCH_DIT) return 11 + 10 * d->n_dual;
+  return 10 + 20 * d->n_dual + 6 * d->n_single;
+}
+
+long long featfix_token_row(const featfix_model_desc* d, int b, int n) {
+  if (!d) return -1;
+  const int bm = d->batch * (d->cfg ? 2 : 1);
+  const int nt = d->txt_tokens, ni = img_tokens(*d);
+  if (b < 0 || b >= bm || n < 0 || n >= nt + ni) return -1;
+  return n < nt ? (long long)b * nt + n : (long long)bm * nt + (long long)b * ni + (n - nt);
+}
+
+featfix_status featfix_plan_build(int steps, int n_layers_, const int* refresh, int n_refresh, int draft_order,
+                                  const featfix_site* sites, int n_sites, int mode, unsigned flags,
+                                  unsigned char* kinds, int* k_eff, double* weights) {
+  std::vector<unsigned char> kd;
+  std::vector<int> ke;
+  std::vector<double> wt;
+  std::vector<char> isref;
+  std::string err;
+  featfix_status s = plan_core(steps, n_layers_, refresh, n_refresh, draft_order, sites, n_sites, mode, flags, kd, ke,
+                               wt, isref, err);
+  if (s != FEATFIX_OK) return s;
+  if (kinds) std::memcpy(kinds, kd.data(), kd.size());
+  if (k_eff) std::memcpy(k_eff, ke.data(), ke.size() * sizeof(int));
+  if (weights) std::memcpy(weights, wt.data(), wt.size() * sizeof(double));
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_create(const featfix_model_desc* desc, const void* const* dev_weights, int n_weights,
+                              void* cuda_stream, featfix_ctx** out) {
+  if (!out) return FEATFIX_ERR_INVALID_ARG;
+  *out = nullptr;
+  const std::string why = check_desc(desc);
+  if (!why.empty()) return FEATFIX_ERR_INVALID_ARG;
+  const int nw = featfix_weight_count(desc);
+  if (!dev_weights || n_weights != nw) return FEATFIX_ERR_INVALID_ARG;
+  for (int k = 0; k < nw; ++k)
+    if (!dev_weights[k] || ((uintptr_t)dev_weights[k] & 15)) return FEATFIX_ERR_INVALID_ARG;
+
+  featfix_ctx* ctx = new featfix_ctx();
+  const featfix_model_desc& d = *desc;
+  ctx->d = d;
+  ctx->dt = d.dtype == FEATFIX_DTYPE_BF16 ? BF16 : F32;
+  ctx->es = dsize(ctx->dt);
+  ctx->L = n_layers(d);
+  ctx->Bm = d.batch * (d.cfg ? 2 : 1);
+  ctx->Nt = d.txt_tokens;
+  ctx->Ni = img_tokens(d);
+  ctx->Ntot = ctx->Nt + ctx->Ni;
+  ctx->C = d.hidden;
+  ctx->H = d.heads;
+  ctx->hd = d.head_dim;
+  ctx->M = d.mlp;
+  ctx->P = patch_vol(d);
+  ctx->fin = ctx->P * d.in_ch;
+  ctx->fout = ctx->P * d.out_ch;
+  ctx->T = (long long)ctx->Bm * ctx->Ntot;
+  ctx->E = ctx->T * ctx->C;
+  ctx->gf = d.lat_f > 0 ? d.lat_f / d.patch_t : 1;
+  ctx->gh = d.lat_h / d.patch;
+  ctx->gw = d.lat_w / d.patch;
+  ctx->w.assign(dev_weights, dev_weights + nw);
+  ctx->st = reinterpret_cast<cudaStream_t>(cuda_stream);
+
+  const int es = ctx->es;
+  const long long T = ctx->T, C = ctx->C, M = ctx->M;
+  featfix_status s = FEATFIX_OK;
+  auto A = [&](void** p, size_t bytes) {
+    if (s == FEATFIX_OK) s = alloc(ctx, p, bytes);
+  };
+  A(&ctx->xa, T * C * es);
+  A(&ctx->xb, T * C * es);
+  A(&ctx->xm, T * C * es);
+  A(&ctx->qkv, T * 3 * C * es);
+  A(&ctx->att, T * C * es);
+  A(&ctx->u1, T * C * es);
+  A(&ctx->big, T * (C + M) * es);
+  A(&ctx->patches, (size_t)ctx->Bm * ctx->Ni * ctx->fin * es);
+  A((void**)&ctx->mod_a, (size_t)ctx->Bm * 6 * C * 4);
+  A((void**)&ctx->mod_b, (size_t)ctx->Bm * 6 * C * 4);
+  A((void**)&ctx->cvec, (size_t)ctx->Bm * C * 4);
+  A((void**)&ctx->csilu, (size_t)ctx->Bm * C * 4);
+  A((void**)&ctx->sinus, 256 * 4);
+  A((void**)&ctx->thid, C * 4);
+  A((void**)&ctx->temb, C * 4);
+  A((void**)&ctx->mout, (size_t)ctx->Bm * ctx->Ni * ctx->fout * 4);
+  if (d.arch == FEATFIX_ARCH_DIT) A(&ctx->pos, (size_t)ctx->Bm * ctx->Ni * C * es);
+  if (d.arch == FEATFIX_ARCH_MMDIT && d.rope_dims) A((void**)&ctx->rope, (size_t)ctx->Ni * (ctx->hd / 2) * sizeof(float2));
+  if (s != FEATFIX_OK) {
+    free_all(ctx);
+    delete ctx;
+    return s;
+  }
+  if (d.arch == FEATFIX_ARCH_DIT && launch_pos2d(ctx->dt, ctx->pos, ctx->Bm, ctx->gh, ctx->gw, ctx->C, ctx->st) != cudaSuccess)
+    s = FEATFIX_ERR_CUDA;
+  if (ctx->rope) {
+    std::vector<float2> tab = rope_table_host(d, ctx->hd);
+    if (cudaMemcpyAsync(ctx->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice, ctx->st) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(ctx->st) != cudaSuccess)
+      s = FEATFIX_ERR_CUDA;
+  }
+  if (s != FEATFIX_OK) {
+    free_all(ctx);
+    delete ctx;
+    return s;
+  }
+  *out = ctx;
+  return FEATFIX_OK;
+}
+
+void featfix_destroy(featfix_ctx* ctx) {
+  if (!ctx) return;
+  cudaStreamSynchronize(ctx->st);
+  free_all(ctx);
+  delete ctx;
+}
+
+featfix_status featfix_set_schedule(featfix_ctx* ctx, int steps, const int* refresh, int n_refresh, int draft_order,
+                                    const featfix_site* sites, int n_sites, int mode, unsigned flags) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  std::vector<unsigned char> kd;
+  std::vector<int> ke;
+  std::vector<double> wt;
+  std::vector<char> isref;
+  std::string err;
+  featfix_status s = plan_core(steps, ctx->L, refresh, n_refresh, draft_order, sites, n_sites, mode, flags, kd, ke, wt,
+                               isref, err);
+  if (s != FEATFIX_OK) return fail(ctx, s, err);
+  if (ctx->d.sampler == FEATFIX_SAMPLER_DDIM && (1000 % steps != 0))
+    return fail(ctx, FEATFIX_ERR_UNSUPPORTED, "DDIM needs steps dividing 1000");
+  cudaStreamSynchronize(ctx->st);
+  const int S = draft_order + 1;
+  if (ctx->ring && ctx->S != S) {
+    cudaFree(ctx->ring);
+    ctx->ring = nullptr;
+  }
+  if (!ctx->ring && mode != FEATFIX_MODE_VANILLA) {
+    s = alloc(ctx, &ctx->ring, (size_t)ctx->L * S * ctx->E * ctx->es);
+    if (s != FEATFIX_OK) return s;
+  }
+  ctx->S = S;
+  const int nlog = std::max(n_sites, 1);
+  if (nlog > ctx->max_logs) {
+    if (ctx->dsums) cudaFree(ctx->dsums);
+    ctx->dsums = nullptr;
+    s = alloc(ctx, (void**)&ctx->dsums, (size_t)nlog * 4 * sizeof(double));
+    if (s != FEATFIX_OK) return s;
+    ctx->max_logs = nlog;
+  }
+  const size_t need = verify_workspace_bytes(ctx->E);
+  if (need > ctx->vws_bytes) {
+    if (ctx->vws) cudaFree(ctx->vws);
+    ctx->vws = nullptr;
+    s = alloc(ctx, &ctx->vws, need);
+    if (s != FEATFIX_OK) return s;
+    ctx->vws_bytes = need;
+  }
+  ctx->kinds.swap(kd);
+  ctx->keff.swap(ke);
+  ctx->wts.swap(wt);
+  ctx->isref.swap(isref);
+  ctx->steps = steps;
+  ctx->K = draft_order;
+  ctx->mode = mode;
+  ctx->flags = flags;
+  ctx->sched = true;
+  ctx->next_step = 0;
+  ctx->cnt = {0, 0, 0, 0};
+  ctx->log_sites.clear();
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_get_plan(featfix_ctx* ctx, unsigned char* kinds, int* k_eff, double* weights) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (!ctx->sched) return fail(ctx, FEATFIX_ERR_STATE, "no schedule");
+  if (kinds) std::memcpy(kinds, ctx->kinds.data(), ctx->kinds.size());
+  if (k_eff) std::memcpy(k_eff, ctx->keff.data(), ctx->keff.size() * sizeof(int));
+  if (weights) std::memcpy(weights, ctx->wts.data(), ctx->wts.size() * sizeof(double));
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_step(featfix_ctx* ctx, float* latent, int i, const void* cond) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (!latent || !cond) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "null latent or cond");
+  if (!ctx->sched) return fail(ctx, FEATFIX_ERR_STATE, "featfix_set_schedule first");
+  if (i != 0 && i != ctx->next_step) return fail(ctx, FEATFIX_ERR_STATE, "step out of order");
+  if (i >= ctx->steps) return fail(ctx, FEATFIX_ERR_STATE, "step beyond the schedule");
+  if (i == 0) {
+    ctx->head = ctx->S - 1;
+    ctx->count = 0;
+    ctx->cnt = {0, 0, 0, 0};
+    ctx->log_sites.clear();
+  }
+  const int L = ctx->L;
+  const bool refresh = ctx->isref[i] != 0;
+  const bool vanilla = ctx->mode == FEATFIX_MODE_VANILLA;
+  const size_t bytes = (size_t)ctx->E * ctx->es;
+  featfix_status s = conditioning(ctx, model_time(ctx, i), cond);
+  if (s != FEATFIX_OK) return s;
+  void* x = ctx->xa;
+  void* y = ctx->xb;
+  s = embed(ctx, latent, cond, x);
+  if (s != FEATFIX_OK) return s;
+  const int new_slot = (ctx->head + 1) % ctx->S;
+  const int nt = ctx->keff[i] + 1;
+  float wf[4];
+  for (int j = 0; j < 4; ++j) wf[j] = (float)ctx->wts[(size_t)i * 4 + j];
+  for (int l = 0; l < L; ++l) {
+    for (auto& cp : ctx->caps)
+      if (cp.step == i && cp.layer == l && cp.in) FF_CK(cudaMemcpyAsync(cp.in, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
+    const unsigned char kind = ctx->kinds[(size_t)i * L + l];
+    if (kind == FEATFIX_PLAN_EXACT) {
+      void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, new_slot) : nullptr;
+      s = exact_block(ctx, l, x, y, hist);
+      if (s != FEATFIX_OK) return s;
+      std::swap(x, y);
+    } else if (kind == FEATFIX_PLAN_DRAFT) {
+      KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
+      FF_CK(launch_draft(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
+    } else {
+      s = exact_block(ctx, l, x, y, nullptr);
+      if (s != FEATFIX_OK) return s;
+      ctx->cnt.paid_checks++;
+      if (ctx->mode != FEATFIX_MODE_EXACT_ONLY) {
+        const int slot = (int)ctx->log_sites.size();
+        if (slot >= ctx->max_logs) return fail(ctx, FEATFIX_ERR_STATE, "log overflow");
+        const int wr = ctx->mode == FEATFIX_MODE_VERIFY ? 1 : 0;
+        KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 2 + wr) * bytes);
+        FF_CK(launch_verify(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, y, ctx->E, wr, ctx->dsums + 4 * slot, ctx->vws,
+                            ctx->st));
+        ctx->log_sites.push_back({i, l});
+      }
+      if (ctx->mode != FEATFIX_MODE_VERIFY) {
+        std::swap(x, y);
+        ctx->cnt.forwarded++;
+      }
+    }
+    for (auto& cp : ctx->caps)
+      if (cp.step == i && cp.layer == l && cp.out) FF_CK(cudaMemcpyAsync(cp.out, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
+  }
+  if (refresh && !vanilla) {
+    ctx->head = new_slot;
+    ctx->count = std::min(ctx->count + 1, ctx->S);
+  }
+  if (refresh || vanilla) ctx->cnt.refresh_steps++;
+  s = finish_step(ctx, i, x, latent);
+  if (s != FEATFIX_OK) return s;
+  ctx->cnt.steps_done = i + 1;
+  ctx->next_step = i + 1;
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_sample(featfix_ctx* ctx, unsigned long long seed, int steps, const void* cond,
+                              float* latent_out) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (!ctx->sched) return fail(ctx, FEATFIX_ERR_STATE, "featfix_set_schedule first");
+  if (steps != ctx->steps) return fail(ctx, FEATFIX_ERR_SCHEDULE, "steps differ from the schedule");
+  if (!latent_out || !cond) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "null latent or cond");
+  const auto& d = ctx->d;
+  const long long n = (long long)d.batch * d.in_ch * (d.lat_f > 0 ? d.lat_f : 1) * d.lat_h * d.lat_w;
+  {
+    KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+    FF_CK(launch_noise(seed, latent_out, n, ctx->st));
+  }
+  for (int i = 0; i < steps; ++i) {
+    featfix_status s = featfix_step(ctx, latent_out, i, cond);
+    if (s != FEATFIX_OK) return s;
+  }
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_sample_host(featfix_ctx* ctx, unsigned long long seed, int steps, const void* cond_host,
+                                   float* latent_out_host) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (!cond_host || !latent_out_host) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "null host buffer");
+  const auto& d = ctx->d;
+  const size_t nlat = (size_t)d.batch * d.in_ch * (d.lat_f > 0 ? d.lat_f : 1) * d.lat_h * d.lat_w;
+  const size_t cbytes = d.arch == FEATFIX_ARCH_DIT ? (size_t)ctx->Bm * sizeof(int)
+                                                    : (size_t)ctx->Bm * ctx->Nt * ctx->C * sizeof(float);
+  featfix_status s = FEATFIX_OK;
+  if (!ctx->h_latent) s = alloc(ctx, (void**)&ctx->h_latent, nlat * sizeof(float));
+  if (s == FEATFIX_OK && !ctx->h_cond) s = alloc(ctx, &ctx->h_cond, cbytes);
+  if (s != FEATFIX_OK) return s;
+  FF_CK(cudaMemcpyAsync(ctx->h_cond, cond_host, cbytes, cudaMemcpyHostToDevice, ctx->st));
+  s = featfix_sample(ctx, seed, steps, ctx->h_cond, ctx->h_latent);
+  if (s != FEATFIX_OK) return s;
+  FF_CK(cudaMemcpyAsync(latent_out_host, ctx->h_latent, nlat * sizeof(float), cudaMemcpyDeviceToHost, ctx->st));
+  FF_CK(cudaStreamSynchronize(ctx->st));
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_get_log(featfix_ctx* ctx, featfix_site_log* out, int cap, int* n, featfix_counters* counters) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  FF_CK(cudaStreamSynchronize(ctx->st));
+  const unsigned int wd = gemm_tc_watchdog_take();
+  if (wd) return fail(ctx, FEATFIX_ERR_CUDA, "tensor-core GEMM watchdog fired (code " + std::to_string(wd) + ")");
+  const int avail = (int)ctx->log_sites.size();
+  if (n) *n = avail;
+  if (counters) *counters = ctx->cnt;
+  const int k = std::min(std::max(cap, 0), avail);
+  if (k > 0 && out) {
+    std::vector<double> sums((size_t)k * 4);
+    FF_CK(cudaMemcpy(sums.data(), ctx->dsums, sums.size() * sizeof(double), cudaMemcpyDeviceToHost));
+    for (int j = 0; j < k; ++j) {
+      const double* q = &sums[(size_t)j * 4];
+      out[j].step = ctx->log_sites[j].first;
+      out[j].layer = ctx->log_sites[j].second;
+      out[j].rel_l1 = q[0] / (q[1] + 1e-8);
+      out[j].rel_l2 = std::sqrt(q[2]) / (std::sqrt(q[3]) + 1e-8);
+      out[j].norm_l1_f = q[1];
+      out[j].norm_l2_f = std::sqrt(q[3]);
+    }
+  }
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_debug_capture(featfix_ctx* ctx, int step, int layer, void* dev_in, void* dev_out) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (step < 0) {
+    ctx->caps.clear();
+    return FEATFIX_OK;
+  }
+  if (layer < 0 || layer >= ctx->L || (!dev_in && !dev_out)) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "bad capture");
+  if (ctx->caps.size() >= 32) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "too many captures");
+  ctx->caps.push_back({step, layer, dev_in, dev_out});
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_debug_block(featfix_ctx* ctx, int step, int layer, const void* dev_in, void* dev_out,
+                                   const void* cond) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (!ctx->sched) return fail(ctx, FEATFIX_ERR_STATE, "featfix_set_schedule first");
+  if (step < 0 || step >= ctx->steps || layer < 0 || layer >= ctx->L || !dev_in || !dev_out || !cond)
+    return fail(ctx, FEATFIX_ERR_INVALID_ARG, "bad debug block request");
+  featfix_status s = conditioning(ctx, model_time(ctx, step), cond);
+  if (s != FEATFIX_OK) return s;
+  return exact_block(ctx, layer, dev_in, dev_out, nullptr);
+}
+
+featfix_status featfix_kernel_timing(featfix_ctx* ctx, int kclass, int on) {
+  if (!ctx || kclass < 0 || kclass >= NKCLASS) return FEATFIX_ERR_INVALID_ARG;
+  FF_CK(cudaStreamSynchronize(ctx->st));
+  timing_drain(ctx);
+  ctx->timing[kclass] = on != 0;
+  ctx->tms[kclass] = 0;
+  ctx->twork[kclass] = 0;
+  ctx->tcount[kclass] = 0;
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_kernel_time(featfix_ctx* ctx, int kclass, double* ms, long long* launches, double* work) {
+  if (!ctx || kclass < 0 || kclass >= NKCLASS) return FEATFIX_ERR_INVALID_ARG;
+  FF_CK(cudaStreamSynchronize(ctx->st));
+  timing_drain(ctx);
+  if (ms) *ms = ctx->tms[kclass];
+  if (launches) *launches = ctx->tcount[kclass];
+  if (work) *work = ctx->twork[kclass];
+  return FEATFIX_OK;
+}
+
+}  // extern "C"

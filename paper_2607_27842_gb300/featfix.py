@@ -75,6 +75,7 @@ SIGNATURES = {
     "featfix_token_row": (_LL, [_P(ModelDesc), _I, _I]),
     "featfix_kernel_timing": (_I, [_VP, _I, _I]),
     "featfix_kernel_time": (_I, [_VP, _I, _P(_D), _P(_LL), _P(_D)]),
+    "featfix_launch_count": (_LL, []),
     "featfix_last_error": (ctypes.c_char_p, [_VP]),
     "featfix_status_string": (ctypes.c_char_p, [_I]),
     "featfix_destroy": (None, [_VP]),
@@ -298,6 +299,10 @@ def featfix_kernel_time(ctx, kclass):
     ms, n, work = _D(0), _LL(0), _D(0)
     _check(lib().featfix_kernel_time(ctx, k, ctypes.byref(ms), ctypes.byref(n), ctypes.byref(work)), ctx)
     return ms.value, n.value, work.value
+
+
+def featfix_launch_count():
+    return int(lib().featfix_launch_count())
 
 
 def featfix_destroy(ctx):

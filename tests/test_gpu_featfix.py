@@ -1,0 +1,204 @@
+"""The whole cached sampling path through the C ABI against the oracle, plus
+the paper's invariants checked bitwise on the GPU (Eq. 5's local reset,
+Exact-only == FeatFix, Verify == no sites, all-refresh == vanilla) and
+run-to-run determinism."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import schedule as osched
+from paper_2607_27842_gb300 import featfix as ff, synthetic as syn
+
+from .gpu_helpers import Case, rel_l2, tol_block, tol_latent
+
+pytestmark = pytest.mark.gpu
+
+
+def small_dit_bf16():
+    sh = syn.reduced(syn.SHAPES["dit_xl2"], n_dual=3, hidden=256, heads=4, head_dim=64, mlp=1024, lat_h=16,
+                     lat_w=16, batch=2, n_classes=10)
+    ref = syn.refresh_every(10, 4)
+    return syn.Workload(sh, 10, 2, ref, syn.diagonal_sites(10, 3, ref, 3))
+
+
+def small_flux(dtype="bf16"):
+    sh = syn.reduced(syn.SHAPES["flux"], n_dual=2, n_single=2, hidden=256, heads=2, head_dim=128, mlp=1024,
+                     lat_h=16, lat_w=16, txt_tokens=12, dtype=dtype)
+    ref = syn.refresh_every(8, 3)
+    return syn.Workload(sh, 8, 1, ref, syn.diagonal_sites(8, 4, ref, 2))
+
+
+def small_qwen():
+    sh = syn.reduced(syn.SHAPES["qwen"], n_dual=3, hidden=256, heads=2, head_dim=128, mlp=1024, lat_h=16, lat_w=16,
+                     txt_tokens=7)
+    ref = syn.refresh_every(9, 3)
+    return syn.Workload(sh, 9, 2, ref, syn.diagonal_sites(9, 3, ref, 3))
+
+
+def small_hunyuan():
+    sh = syn.reduced(syn.SHAPES["hunyuan"], n_dual=2, hidden=256, heads=2, head_dim=128, mlp=1024, lat_f=3,
+                     lat_h=8, lat_w=12, txt_tokens=5)
+    ref = syn.refresh_every(7, 3)
+    return syn.Workload(sh, 7, 1, ref, syn.diagonal_sites(7, 2, ref, 2))
+
+
+WORKLOADS = {
+    "tiny": lambda: syn.workload("tiny"),
+    "dit_bf16": small_dit_bf16,
+    "flux_bf16": small_flux,
+    "flux_f32": lambda: small_flux("f32"),
+    "qwen_bf16": small_qwen,
+    "hunyuan_bf16": small_hunyuan,
+}
+
+
+@pytest.fixture(params=list(WORKLOADS))
+def case(request, cuda):
+    c = Case(WORKLOADS[request.param]())
+    yield c
+    c.close()
+
+
+def test_sample_matches_oracle(case):
+    """Free-running cached trajectory: final latent, logs and accounting."""
+    case.schedule("featfix")
+    lat = case.sample(seed=1)
+    logs, cnt = ff.featfix_get_log(case.ctx)
+    x_ref, logs_ref, cnt_ref = case.oracle_run("featfix", seed=1)
+    err = rel_l2(lat.cpu().numpy(), x_ref)
+    assert err < tol_latent(case.sh), err
+    assert {k: cnt[k] for k in cnt_ref} == cnt_ref
+    assert cnt["steps_done"] == case.wl.steps
+    assert [(e["step"], e["layer"]) for e in logs] == [(e["step"], e["layer"]) for e in logs_ref]
+    for g, r in zip(logs, logs_ref):
+        assert g["rel_l1"] == pytest.approx(r["rel_l1"], rel=0.05 if case.sh.dtype == "bf16" else 1e-3)
+        assert g["rel_l2"] == pytest.approx(r["rel_l2"], rel=0.05 if case.sh.dtype == "bf16" else 1e-3)
+
+
+def test_blocks_teacher_forced(case):
+    """Every block of the trajectory on the GPU's own incoming state: exact
+    blocks vs B_l (Eq. 1), drafts vs Eq. 2 over the GPU's refresh increments."""
+    wl, sh = case.wl, case.sh
+    case.schedule("featfix")
+    L = sh.n_layers
+    kinds, keff, _ = ff.featfix_get_plan(case.ctx, wl.steps, L)
+    picks = [(i, l) for i in range(wl.steps) for l in range(L)]
+    if len(picks) > 30:
+        picks = [p for p in picks if kinds[p] != ff.PLAN_DRAFT or p[1] % 3 == 0][:30]
+    bufs = {}
+    for (i, l) in picks:
+        bufs[(i, l)] = (case.act_buffer(), case.act_buffer())
+        ff.featfix_debug_capture(case.ctx, i, l, *bufs[(i, l)])
+    # refresh increments of every layer for the draft checks
+    inc = {}
+    for i in wl.refresh:
+        for l in range(L):
+            if (i, l) not in bufs:
+                bufs[(i, l)] = (case.act_buffer(), case.act_buffer())
+                ff.featfix_debug_capture(case.ctx, i, l, *bufs[(i, l)])
+    case.sample(seed=1)
+    for i in wl.refresh:
+        for l in range(L):
+            u, h = bufs[(i, l)]
+            inc[(i, l)] = case.to_logical(h) - case.to_logical(u)
+    ang = oracle.model.rope_table(sh)
+    for (i, l) in picks:
+        u = case.to_logical(bufs[(i, l)][0])
+        h = case.to_logical(bufs[(i, l)][1])
+        k = kinds[i, l]
+        if k == ff.PLAN_DRAFT:
+            hist = [(s, inc[(s, l)]) for s in sorted([r for r in wl.refresh if r <= i], reverse=True)]
+            ref = oracle.draft.draft(u, hist[:wl.K + 1], i, wl.K)
+            tol = 1e-6 if sh.dtype == "f32" else 8e-3
+        else:
+            ref = oracle.featfix.block_at(case.W64, sh, l, i, wl.steps, u, case.cond64)
+            tol = tol_block(sh)
+        assert rel_l2(h, ref) < tol, (i, l, k, rel_l2(h, ref))
+    ff.featfix_debug_capture(case.ctx, -1, 0, None, None)
+
+
+def test_featfix_site_forwards_exact_output_bitwise(case):
+    """Eq. 5: at a site the forwarded tensor is B_l(u) from the same u."""
+    wl = case.wl
+    case.schedule("featfix")
+    i, l = wl.sites[0]
+    u, h = case.act_buffer(), case.act_buffer()
+    ff.featfix_debug_capture(case.ctx, i, l, u, h)
+    case.sample(seed=3)
+    hf = case.act_buffer()
+    ff.featfix_debug_block(case.ctx, i, l, u, hf, case.cond)
+    torch.cuda.synchronize()
+    assert torch.equal(h, hf)
+
+
+def test_arms_bitwise(case):
+    """Exact-only == FeatFix; Verify == schedule without sites; all-refresh ==
+    vanilla; two runs identical."""
+    wl = case.wl
+    runs = {}
+    for tag, mode, sites, refresh in (("featfix", "featfix", None, None), ("exact_only", "exact_only", None, None),
+                                      ("verify", "verify", None, None), ("nosite", "featfix", (), None),
+                                      ("allref", "featfix", (), tuple(range(wl.steps))),
+                                      ("vanilla", "vanilla", None, None)):
+        case.schedule(mode, refresh=refresh, sites=sites)
+        runs[tag] = case.sample(seed=5).clone()
+        runs[tag + "_log"] = ff.featfix_get_log(case.ctx)
+    assert torch.equal(runs["featfix"], runs["exact_only"])
+    assert torch.equal(runs["verify"], runs["nosite"])
+    assert torch.equal(runs["allref"], runs["vanilla"])
+    assert not torch.equal(runs["featfix"], runs["verify"])
+    n = len(wl.sites)
+    assert runs["featfix_log"][1]["forwarded"] == n and runs["verify_log"][1]["forwarded"] == 0
+    assert runs["exact_only_log"][0] == [] and runs["exact_only_log"][1]["paid_checks"] == n
+    assert runs["vanilla_log"][1]["refresh_steps"] == wl.steps
+    # same state at the first paid check in both arms -> same logged value
+    assert runs["featfix_log"][0][0]["rel_l1"] == runs["verify_log"][0][0]["rel_l1"]
+    case.schedule("featfix")
+    again = case.sample(seed=5)
+    assert torch.equal(again, runs["featfix"])
+    assert ff.featfix_get_log(case.ctx)[0] == runs["featfix_log"][0]
+
+
+def test_call_order_errors(cuda):
+    c = Case(syn.workload("tiny"))
+    try:
+        lat = torch.zeros(c.sh.latent_dims, device=cuda)
+        with pytest.raises(ff.FeatFixError) as e:
+            ff.featfix_step(c.ctx, lat, 0, c.cond)
+        assert e.value.status == ff.ERR_STATE
+        c.schedule("featfix")
+        with pytest.raises(ff.FeatFixError) as e:
+            ff.featfix_step(c.ctx, lat, 3, c.cond)
+        assert e.value.status == ff.ERR_STATE
+        with pytest.raises(ff.FeatFixError) as e:
+            ff.featfix_sample(c.ctx, 1, 9, c.cond, lat)
+        assert e.value.status == ff.ERR_SCHEDULE
+        with pytest.raises(ff.FeatFixError) as e:
+            ff.featfix_set_schedule(c.ctx, 10, (0, 3), 1, ((3, 1),))
+        assert e.value.status == ff.ERR_SCHEDULE
+        # step-wise driving equals featfix_sample
+        c.schedule("featfix")
+        ref = c.sample(seed=4)
+        import oracle as orc
+        x = torch.from_numpy(orc.noise.initial_latent(4, c.sh)).to(cuda)
+        for i in range(c.wl.steps):
+            ff.featfix_step(c.ctx, x, i, c.cond)
+        torch.cuda.synchronize()
+        assert rel_l2(x.cpu().numpy(), ref.cpu().numpy()) < 1e-6
+    finally:
+        c.close()
+
+
+def test_sample_host_matches_device(cuda):
+    c = Case(small_dit_bf16())
+    try:
+        c.schedule("featfix")
+        ref = c.sample(seed=9).cpu()
+        cond_h = c.cond_cpu.pin_memory()
+        out_h = torch.empty(c.sh.latent_dims, dtype=torch.float32).pin_memory()
+        ff.featfix_sample_host(c.ctx, 9, c.wl.steps, cond_h, out_h)
+        assert torch.equal(out_h, ref)
+    finally:
+        c.close()
