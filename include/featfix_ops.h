@@ -46,6 +46,40 @@ FEATFIX_API featfix_status featfix_op_verify(int dtype, void* dev_u, const void*
                                  int n_terms, const void* dev_hf, long long n, int write_draft,
                                  double* dev_sums, void* dev_workspace, size_t ws_bytes, void* stream);
 
+/* featfix_op_verify without any device allocation.  The paper has no
+ * counterpart: this is a deployment convenience.
+ *
+ * Some callers cannot allocate device memory at all: a host application or
+ * plugin framework that owns every byte of the GPU and forbids side
+ * allocations, a memory-budgeted service that plans all device memory up
+ * front, or a latency-critical loop where a cudaMalloc (with its implicit
+ * synchronisation and possible failure) is not acceptable.  For them this
+ * entry point computes exactly what featfix_op_verify computes (same sums,
+ * same deterministic reduction order, same Verify-arm write of h_d) with the
+ * per-cluster partial sums kept in a fixed scratch array of
+ * FEATFIX_VERIFY_NOALLOC_SCRATCH_BYTES (16 KiB) compiled into the library.
+ * The caller still provides dev_u, dev_hist, dev_hf and dev_sums.
+ *
+ *  - No cudaMalloc, cudaFree or other allocating routine is called.  Every
+ *    GPU that loads the library holds the 16 KiB array until the process
+ *    exits.
+ *  - The first call on a device looks up the array's device address (with
+ *    that device current) and caches it; make that first call before any
+ *    stream capture on the device.
+ *  - A call needs featfix_op_verify_workspace(n) bytes of the array (one
+ *    32-byte partial per 8-CTA cluster, at most 4 CTAs per SM); if that is
+ *    more than 16 KiB (a GPU with more than 1024 SMs) the call returns
+ *    FEATFIX_ERR_INVALID_ARG and launches nothing.
+ *  - All calls, on every stream of a device, share the one array, which
+ *    keeps the last call's contents.  Each launch writes every partial it
+ *    reads back, so nothing needs clearing; but calls whose executions
+ *    overlap on the GPU race on the array and may return wrong sums:
+ *    serialise them (one stream, or events between streams).             */
+#define FEATFIX_VERIFY_NOALLOC_SCRATCH_BYTES 16384
+FEATFIX_API featfix_status featfix_op_verify_noalloc(int dtype, void* dev_u, const void* const* dev_hist,
+                                                     const double* w, int n_terms, const void* dev_hf, long long n,
+                                                     int write_draft, double* dev_sums, void* stream);
+
 /* adaLN input of a branch: out[r,:] = LN(x[r,:]) * (1 + scale[b,:]) + shift[b,:]
  * with LN over C columns without affine (eps 1e-6), b = r / rows_per_batch,
  * shift/scale float32 rows of stride mod_stride.  x, out row-major [rows, C]. */

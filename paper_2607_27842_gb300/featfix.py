@@ -82,6 +82,7 @@ SIGNATURES = {
     "featfix_op_draft": (_I, [_I, _VP, _P(_VP), _P(_D), _I, _LL, _VP]),
     "featfix_op_verify_workspace": (ctypes.c_size_t, [_LL]),
     "featfix_op_verify": (_I, [_I, _VP, _P(_VP), _P(_D), _I, _VP, _LL, _I, _VP, _VP, ctypes.c_size_t, _VP]),
+    "featfix_op_verify_noalloc": (_I, [_I, _VP, _P(_VP), _P(_D), _I, _VP, _LL, _I, _VP, _VP]),
     "featfix_op_ln_modulate": (_I, [_I, _VP, _VP, _LL, _I, _VP, _VP, _I, _I, _VP]),
     "featfix_op_gemm": (_I, [_I, _I, _I, _I, _VP, _VP, _VP, _I, _VP, _I, _I, _VP, _VP, _VP, _VP, _VP]),
     "featfix_op_attention": (_I, [_I, _VP, _I, _VP, _I, _I, _I, _I, _I, _I, _VP]),
@@ -334,6 +335,15 @@ def featfix_op_verify(dtype, u, hist, w, hf, sums, workspace, write_draft=False,
     _check(lib().featfix_op_verify(_dt(dtype), _ptr(u), hp, wa, len(hist), _ptr(hf), u.numel(), int(write_draft),
                                    _ptr(sums), _ptr(workspace), workspace.numel() * workspace.element_size(),
                                    _stream_ptr(stream)))
+
+
+def featfix_op_verify_noalloc(dtype, u, hist, w, hf, sums, write_draft=False, stream=None):
+    """featfix_op_verify with the library's fixed scratch array (no device
+    allocation by anyone); see include/featfix_ops.h."""
+    hp = (_VP * len(hist))(*[_ptr(h) for h in hist])
+    wa = (_D * len(hist))(*[float(v) for v in w])
+    _check(lib().featfix_op_verify_noalloc(_dt(dtype), _ptr(u), hp, wa, len(hist), _ptr(hf), u.numel(),
+                                           int(write_draft), _ptr(sums), _stream_ptr(stream)))
 
 
 def featfix_op_ln_modulate(dtype, x, out, rows, C, shift, scale, mod_stride, rows_per_batch, stream=None):
