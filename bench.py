@@ -289,10 +289,12 @@ def main():
     barrier()
 
     # ---- device-resident timed region (kernel-class timing on) ----
-    ff.featfix_kernel_timing(ctx, "gemm", True)
-    ff.featfix_kernel_timing(ctx, "draft", True)
-    ff.featfix_kernel_timing(ctx, "attention", True)
-    ff.featfix_kernel_timing(ctx, "verify", True)
+    timed_classes = ("gemm", "draft", "attention", "verify")
+    for k in timed_classes:
+        ff.featfix_kernel_timing(ctx, k, True)
+    ff.featfix_sample(ctx, 999, wl.steps, cond, lat)      # untimed: rebuilds the graph with timing events
+    for k in timed_classes:
+        ff.featfix_kernel_timing(ctx, k, True)             # zero the counters (graph kept)
     clocks = ClockSampler(local)
     clocks.start()
     l0 = ff.featfix_launch_count()
@@ -306,7 +308,7 @@ def main():
     clk = clocks.stop()
     launches = ff.featfix_launch_count() - l0
     ms = ev0.elapsed_time(ev1)
-    kt = {k: ff.featfix_kernel_time(ctx, k) for k in ("gemm", "draft", "attention", "verify")}
+    kt = {k: ff.featfix_kernel_time(ctx, k) for k in timed_classes}
     for k in kt:
         ff.featfix_kernel_timing(ctx, k, False)
     logs, counters = ff.featfix_get_log(ctx)   # synchronises and checks the watchdog

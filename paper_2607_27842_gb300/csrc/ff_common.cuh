@@ -64,7 +64,7 @@ __device__ __forceinline__ float silu(float x) { return x / (1.0f + expf(-x)); }
 // ---------------------------------------------------------------------------
 struct EpiArgs {
   const void* bias;      // [N] model dtype (nullable)
-  int act;               // 0 identity, 1 GELU(tanh)
+  int act;               // 0 identity, 1 GELU(tanh), 2 SiLU
   int act_col0;          // activation only on columns >= act_col0
   const float* gate;     // gate rows (nullable): gate[b * gate_stride + n]
   int gate_stride;
@@ -136,6 +136,9 @@ __device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N
   if (e.act == 1 && n0 >= e.act_col0) {
 #pragma unroll
     for (int j = 0; j < CH; ++j) v[j] = gelu_tanh(v[j]);
+  } else if (e.act == 2 && n0 >= e.act_col0) {
+#pragma unroll
+    for (int j = 0; j < CH; ++j) v[j] = silu(v[j]);
   }
   if (e.gate) {
     const float* g = e.gate + (size_t)epi_batch(e, m) * e.gate_stride + n0;
@@ -219,9 +222,13 @@ cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int
                           int write_draft, double* sums, void* ws, cudaStream_t s);
 cudaError_t launch_ln_mod(DType dt, const void* x, void* out, long long rows, int C, const float* shift,
                           const float* scale, int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s);
-cudaError_t launch_linear_small(DType wt, const float* x, int B, int K, const void* W, const void* bias, int N,
-                                float* y, int ldy, int silu_in, int silu_out, cudaStream_t s);
-cudaError_t launch_sinusoid(float t, float* out, int dim, cudaStream_t s);
+// Sinusoidal features of S model times (device array) -> [S, 256] in dt.
+cudaError_t launch_sinusoid_table(DType dt, const float* times, int S, void* out, cudaStream_t s);
+// SiLU(temb[s] + y_emb[label_b]) for every (step s, sample b): rows s*B + b of
+// `all` ([S*B, C], dt); rows of steps with need_row[s] >= 0 also go to
+// need[(need_row[s]*B + b)] (gathered table).
+cudaError_t launch_cond_table(DType dt, const float* temb, const void* y_emb, const int* labels, int S, int B, int C,
+                              const int* need_row, void* all, void* need, cudaStream_t s);
 cudaError_t launch_cond_finish(DType wt, const float* e, const void* y_emb, const int* labels, int B, int C,
                                float* c_out, float* csilu_out, cudaStream_t s);
 cudaError_t launch_patchify(DType dt, const float* latent, int B_lat, int B_model, int Cin, int F, int H, int W,

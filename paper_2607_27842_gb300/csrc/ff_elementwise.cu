@@ -1,6 +1,6 @@
 // Bandwidth-bound kernels of the FeatFix denoising step: the draft (Eq. 2),
 // the fused paid check / forward (Eqs. 3-5), adaLN LayerNorm-modulation,
-// conditioning GEMVs, embedding, sampler update and the seeded latent.
+// conditioning tables, embedding, sampler update and the seeded latent.
 #include "ff_common.cuh"
 
 #include <cooperative_groups.h>
@@ -224,10 +224,10 @@ cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int
 
 // ---------------------------------------------------------------------------
 // adaLN branch input: LN(x) (no affine, eps 1e-6) * (1 + scale_b) + shift_b.
-// One warp per row; the row is read three times (mean, variance, output),
-// the re-reads hit L1.
+// One warp per row, the row held in registers (NCH 16-byte vectors per
+// lane): one global read, exact two-pass mean / variance, one write.
 // ---------------------------------------------------------------------------
-template <class T>
+template <class T, int NCH>
 __global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
                                                 const float* __restrict__ shift, const float* __restrict__ scale,
                                                 int mod_stride, int seg_split, int rpb0, int rpb1) {
@@ -237,21 +237,26 @@ __global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __re
   if (r >= rows) return;
   const T* xr = x + r * C;
   const int nv = C / V;
+  float a[NCH][V];
   float s = 0.f;
-  for (int k = lane; k < nv; k += 32) {
-    float a[V];
-    ld16(xr + k * V, a);
 #pragma unroll
-    for (int q = 0; q < V; ++q) s += a[q];
+  for (int j = 0; j < NCH; ++j) {
+    const int k = lane + 32 * j;
+    if (k < nv) {
+      ld16(xr + k * V, a[j]);
+#pragma unroll
+      for (int q = 0; q < V; ++q) s += a[j][q];
+    }
   }
   s = warp_sum(s);
   const float mean = s / C;
   float ss = 0.f;
-  for (int k = lane; k < nv; k += 32) {
-    float a[V];
-    ld16(xr + k * V, a);
 #pragma unroll
-    for (int q = 0; q < V; ++q) { const float d = a[q] - mean; ss += d * d; }
+  for (int j = 0; j < NCH; ++j) {
+    if (lane + 32 * j < nv) {
+#pragma unroll
+      for (int q = 0; q < V; ++q) { const float d = a[j][q] - mean; ss += d * d; }
+    }
   }
   ss = warp_sum(ss);
   const float rstd = rsqrtf(ss / C + 1e-6f);
@@ -259,165 +264,103 @@ __global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __re
   const float* sh = shift + (size_t)b * mod_stride;
   const float* sc = scale + (size_t)b * mod_stride;
   T* orow = out + r * C;
-  for (int k = lane; k < nv; k += 32) {
-    float a[V];
-    ld16(xr + k * V, a);
 #pragma unroll
-    for (int q = 0; q < V; ++q) {
-      const int c = k * V + q;
-      a[q] = (a[q] - mean) * rstd * (1.0f + sc[c]) + sh[c];
+  for (int j = 0; j < NCH; ++j) {
+    const int k = lane + 32 * j;
+    if (k < nv) {
+      float o[V];
+#pragma unroll
+      for (int q = 0; q < V; q += 4) {
+        const float4 s4 = *reinterpret_cast<const float4*>(sh + k * V + q);
+        const float4 c4 = *reinterpret_cast<const float4*>(sc + k * V + q);
+        o[q] = (a[j][q] - mean) * rstd * (1.0f + c4.x) + s4.x;
+        o[q + 1] = (a[j][q + 1] - mean) * rstd * (1.0f + c4.y) + s4.y;
+        o[q + 2] = (a[j][q + 2] - mean) * rstd * (1.0f + c4.z) + s4.z;
+        o[q + 3] = (a[j][q + 3] - mean) * rstd * (1.0f + c4.w) + s4.w;
+      }
+      st16(orow + k * V, o);
     }
-    st16(orow + k * V, a);
   }
+}
+
+template <class T>
+static cudaError_t ln_mod_t(const void* x, void* out, long long rows, int C, const float* shift, const float* scale,
+                            int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s) {
+  constexpr int V = VecN<T>::n;
+  const int nch = (C / V + 31) / 32;
+  const unsigned grid = (unsigned)((rows + 7) / 8);
+  const T* xp = (const T*)x;
+  T* op = (T*)out;
+#define FF_LN_CASE(n) \
+  case n: k_ln_mod<T, n><<<grid, 256, 0, s>>>(xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break;
+  switch (nch) {
+    FF_LN_CASE(1) FF_LN_CASE(2) FF_LN_CASE(3) FF_LN_CASE(4) FF_LN_CASE(5) FF_LN_CASE(6)
+    FF_LN_CASE(8) FF_LN_CASE(12) FF_LN_CASE(16)
+    default:
+      if (nch <= 8) { k_ln_mod<T, 8><<<grid, 256, 0, s>>>(xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      if (nch <= 12) { k_ln_mod<T, 12><<<grid, 256, 0, s>>>(xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      if (nch <= 16) { k_ln_mod<T, 16><<<grid, 256, 0, s>>>(xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      return cudaErrorInvalidValue;
+  }
+#undef FF_LN_CASE
+  return launched();
 }
 
 cudaError_t launch_ln_mod(DType dt, const void* x, void* out, long long rows, int C, const float* shift,
                           const float* scale, int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  const unsigned grid = (unsigned)((rows + 7) / 8);
-  if (dt == F32)
-    k_ln_mod<float><<<grid, 256, 0, s>>>((const float*)x, (float*)out, rows, C, shift, scale, mod_stride, seg_split,
-                                         rpb0, rpb1);
-  else
-    k_ln_mod<bf16><<<grid, 256, 0, s>>>((const bf16*)x, (bf16*)out, rows, C, shift, scale, mod_stride, seg_split,
-                                        rpb0, rpb1);
+  if (((uintptr_t)shift & 15) || ((uintptr_t)scale & 15) || (mod_stride & 3)) return cudaErrorInvalidValue;
+  if (dt == F32) return ln_mod_t<float>(x, out, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1, s);
+  return ln_mod_t<bf16>(x, out, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1, s);
+}
+
+// Sinusoidal features of every model time: row s = [cos(t_s f_k) | sin(t_s f_k)].
+template <class T>
+__global__ void k_sinusoid_table(const float* __restrict__ times, int S, T* __restrict__ out) {
+  const int s = blockIdx.x;
+  if (s >= S) return;
+  const double t = (double)times[s];
+  for (int k = threadIdx.x; k < 128; k += blockDim.x) {
+    const double f = exp(-log(10000.0) * (double)k / 128.0);
+    out[(size_t)s * 256 + k] = from_f<T>((float)cos(t * f));
+    out[(size_t)s * 256 + 128 + k] = from_f<T>((float)sin(t * f));
+  }
+}
+
+cudaError_t launch_sinusoid_table(DType dt, const float* times, int S, void* out, cudaStream_t s) {
+  if (S <= 0) return cudaSuccess;
+  if (dt == F32) k_sinusoid_table<float><<<S, 128, 0, s>>>(times, S, (float*)out);
+  else k_sinusoid_table<bf16><<<S, 128, 0, s>>>(times, S, (bf16*)out);
   return launched();
 }
 
-// ---------------------------------------------------------------------------
-// Conditioning GEMV for a handful of rows: y[b, n] = f(sum_k W[n,k] g(x[b,k]) + bias[n]).
-// x sits in shared memory; each warp produces 4 outputs at a time so one
-// shared-memory read of x feeds 4 weight rows.
-// ---------------------------------------------------------------------------
-constexpr int LS_WARPS = 8;
-constexpr int LS_NPW = 4;
-
-template <class TW, int BMAX>
-__global__ void __launch_bounds__(LS_WARPS * 32) k_linear_small(const float* __restrict__ x, int B, int K,
-                                                                const TW* __restrict__ W, const TW* __restrict__ bias,
-                                                                int N, float* __restrict__ y, int ldy, int silu_in,
-                                                                int silu_out) {
-  extern __shared__ float xs[];
-  for (int i = threadIdx.x; i < B * K; i += blockDim.x) {
-    const float v = x[i];
-    xs[i] = silu_in ? silu(v) : v;
-  }
-  __syncthreads();
-  constexpr int V = VecN<TW>::n;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nv = K / V;
-  for (int n0 = (blockIdx.x * LS_WARPS + warp) * LS_NPW; n0 < N; n0 += gridDim.x * LS_WARPS * LS_NPW) {
-    float acc[LS_NPW][BMAX];
-#pragma unroll
-    for (int a = 0; a < LS_NPW; ++a)
-#pragma unroll
-      for (int b = 0; b < BMAX; ++b) acc[a][b] = 0.f;
-    for (int k = lane; k < nv; k += 32) {
-      float wv[LS_NPW][V];
-#pragma unroll
-      for (int a = 0; a < LS_NPW; ++a) {
-        if (n0 + a < N) ld16(W + (size_t)(n0 + a) * K + k * V, wv[a]);
-        else {
-#pragma unroll
-          for (int q = 0; q < V; ++q) wv[a][q] = 0.f;
-        }
-      }
-#pragma unroll
-      for (int b = 0; b < BMAX; ++b) {
-        if (b < B) {
-          const float* xb = xs + b * K + k * V;
-#pragma unroll
-          for (int q = 0; q < V; ++q) {
-            const float xv = xb[q];
-#pragma unroll
-            for (int a = 0; a < LS_NPW; ++a) acc[a][b] = fmaf(wv[a][q], xv, acc[a][b]);
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int a = 0; a < LS_NPW; ++a) {
-#pragma unroll
-      for (int b = 0; b < BMAX; ++b) {
-        if (b < B) {
-          const float t = warp_sum(acc[a][b]);
-          if (lane == 0 && n0 + a < N) {
-            float v = t + (bias ? to_f(bias[n0 + a]) : 0.f);
-            y[(size_t)b * ldy + n0 + a] = silu_out ? silu(v) : v;
-          }
-        }
-      }
-    }
-  }
-}
-
-template <class TW, int BMAX>
-static cudaError_t linear_small_t(const float* x, int B, int K, const void* W, const void* bias, int N, float* y,
-                                  int ldy, int silu_in, int silu_out, cudaStream_t s) {
-  const size_t smem = (size_t)B * K * sizeof(float);
-  auto fn = k_linear_small<TW, BMAX>;
-  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  int blocks = (N + LS_WARPS * LS_NPW - 1) / (LS_WARPS * LS_NPW);
-  if (blocks > num_sms() * 2) blocks = num_sms() * 2;
-  fn<<<blocks, LS_WARPS * 32, smem, s>>>(x, B, K, (const TW*)W, (const TW*)bias, N, y, ldy, silu_in, silu_out);
-  return launched();
-}
-
-cudaError_t launch_linear_small(DType wt, const float* x, int B, int K, const void* W, const void* bias, int N,
-                                float* y, int ldy, int silu_in, int silu_out, cudaStream_t s) {
-  if ((size_t)B * K * sizeof(float) > 200 * 1024) return cudaErrorInvalidValue;
-  if (wt == F32) {
-    if (K % 4) return cudaErrorInvalidValue;
-    if (B <= 2) return linear_small_t<float, 2>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
-    if (B <= 8) return linear_small_t<float, 8>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
-    if (B <= 16) return linear_small_t<float, 16>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
-    if (B <= 32) return linear_small_t<float, 32>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
-  } else {
-    if (K % 8) return cudaErrorInvalidValue;
-    if (B <= 2) return linear_small_t<bf16, 2>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
-    if (B <= 8) return linear_small_t<bf16, 8>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
-    if (B <= 16) return linear_small_t<bf16, 16>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
-    if (B <= 32) return linear_small_t<bf16, 32>(x, B, K, W, bias, N, y, ldy, silu_in, silu_out, s);
-  }
-  return cudaErrorInvalidValue;
-}
-
-// Sinusoidal timestep features: [cos(t f_k) | sin(t f_k)], f_k = 10000^(-k/half).
-__global__ void k_sinusoid(float t, float* out, int dim) {
-  const int half = dim / 2;
-  for (int k = threadIdx.x; k < half; k += blockDim.x) {
-    const double f = exp(-log(10000.0) * (double)k / (double)half);
-    const double a = (double)t * f;
-    out[k] = (float)cos(a);
-    out[k + half] = (float)sin(a);
-  }
-}
-
-cudaError_t launch_sinusoid(float t, float* out, int dim, cudaStream_t s) {
-  k_sinusoid<<<1, 128, 0, s>>>(t, out, dim);
-  return launched();
-}
-
-// c[b] = e (+ y_emb[label_b]); csilu = SiLU(c).
-template <class TW>
-__global__ void k_cond_finish(const float* __restrict__ e, const TW* __restrict__ y_emb, const int* __restrict__ labels,
-                              int B, int C, float* __restrict__ c_out, float* __restrict__ csilu) {
-  const int b = blockIdx.x;
+// SiLU(c) of every (step, sample): c = temb[step] (+ y_emb[label]).
+template <class T>
+__global__ void k_cond_table(const float* __restrict__ temb, const T* __restrict__ y_emb, const int* __restrict__ labels,
+                             int S, int B, int C, const int* __restrict__ need_row, T* __restrict__ all,
+                             T* __restrict__ need) {
+  const int row = blockIdx.x;  // s * B + b
+  const int s = row / B, b = row % B;
+  if (s >= S) return;
+  const int nr = need_row ? need_row[s] : -1;
   for (int k = threadIdx.x; k < C; k += blockDim.x) {
-    float v = e[k];
+    float v = temb[(size_t)s * C + k];
     if (y_emb) v += to_f(y_emb[(size_t)labels[b] * C + k]);
-    c_out[(size_t)b * C + k] = v;
-    csilu[(size_t)b * C + k] = silu(v);
+    const T o = from_f<T>(silu(v));
+    all[(size_t)row * C + k] = o;
+    if (nr >= 0) need[((size_t)nr * B + b) * C + k] = o;
   }
 }
 
-cudaError_t launch_cond_finish(DType wt, const float* e, const void* y_emb, const int* labels, int B, int C,
-                               float* c_out, float* csilu_out, cudaStream_t s) {
-  if (wt == F32)
-    k_cond_finish<float><<<B, 256, 0, s>>>(e, (const float*)y_emb, labels, B, C, c_out, csilu_out);
+cudaError_t launch_cond_table(DType dt, const float* temb, const void* y_emb, const int* labels, int S, int B, int C,
+                              const int* need_row, void* all, void* need, cudaStream_t s) {
+  if (S <= 0) return cudaSuccess;
+  if (dt == F32)
+    k_cond_table<float><<<S * B, 256, 0, s>>>(temb, (const float*)y_emb, labels, S, B, C, need_row, (float*)all,
+                                              (float*)need);
   else
-    k_cond_finish<bf16><<<B, 256, 0, s>>>(e, (const bf16*)y_emb, labels, B, C, c_out, csilu_out);
+    k_cond_table<bf16><<<S * B, 256, 0, s>>>(temb, (const bf16*)y_emb, labels, S, B, C, need_row, (bf16*)all,
+                                             (bf16*)need);
   return launched();
 }
 

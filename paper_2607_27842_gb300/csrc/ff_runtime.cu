@@ -1,7 +1,8 @@
 // Host runtime of the FeatFix cached denoising path and the C ABI of
 // include/featfix.h: context and workspace, the fixed schedule (Section 3.3),
 // the draft weights of Eq. 2, the per-step block loop (Eqs. 1-5), logs,
-// accounting, debug capture and kernel timing.
+// accounting, debug capture, kernel timing and the CUDA-graph replay of
+// whole trajectories.
 #include "featfix.h"
 #include "featfix_ops.h"
 #include "ff_common.cuh"
@@ -40,22 +41,49 @@ struct featfix_ctx {
   long long T, E;
   int gf, gh, gw;
   std::vector<const void*> w;
-  cudaStream_t st;
+  cudaStream_t user_st = nullptr;  // caller's stream
+  cudaStream_t cap_st = nullptr;   // private stream used only to capture graphs
+  cudaStream_t st = nullptr;       // stream work is issued on (user_st, or cap_st while capturing)
 
+  // activations
   void *xa = nullptr, *xb = nullptr, *xm = nullptr, *qkv = nullptr, *att = nullptr, *u1 = nullptr, *big = nullptr;
   void *patches = nullptr, *pos = nullptr;
-  float *mod_a = nullptr, *mod_b = nullptr, *cvec = nullptr, *csilu = nullptr, *sinus = nullptr, *thid = nullptr,
-        *temb = nullptr, *mout = nullptr;
+  float* mout = nullptr;
   float2* rope = nullptr;
+  // refresh history
   void* ring = nullptr;
   int S = 0;
+  // modulation: concatenated block weights and the per-trajectory tables
+  void* wmod = nullptr;
+  void* bmod = nullptr;
+  long long Nblk = 0;
+  std::vector<long long> moff;      // column of block l, stream s (0 image / only, 1 text) at 2l + s
+  float* d_times = nullptr;         // [steps] model times
+  int* d_need = nullptr;            // [steps] row block in the block-mod table, -1 if none
+  std::vector<int> need_row;
+  int n_need = 0;
+  void* sin_tab = nullptr;          // [steps, 256]
+  void* thid_tab = nullptr;         // [steps, C]
+  float* temb_tab = nullptr;        // [steps, C]
+  void* cs_all = nullptr;           // [steps * Bm, C]   SiLU(c)
+  void* cs_need = nullptr;          // [n_need * Bm, C]  gathered rows of steps with exact blocks
+  float* bmodtab = nullptr;         // [(n_need + 1) * Bm, Nblk]; the last row block is for featfix_debug_block
+  float* fmodtab = nullptr;         // [steps * Bm, 2C]
+  int mod_row_override = -1;
+  // logs
   double* dsums = nullptr;
   int max_logs = 0;
   void* vws = nullptr;
   size_t vws_bytes = 0;
-  float* h_latent = nullptr;  // device buffers of featfix_sample_host
+  // device copies of featfix_sample's inputs (fixed addresses for the graph)
+  float* g_lat = nullptr;
+  void* g_cond = nullptr;
+  size_t cond_bytes = 0;
+  long long lat_elems = 0;
+  float* h_latent = nullptr;        // featfix_sample_host output staging
   void* h_cond = nullptr;
 
+  // schedule
   bool sched = false;
   int steps = 0, K = 0, mode = 0;
   unsigned flags = 0;
@@ -64,12 +92,21 @@ struct featfix_ctx {
   std::vector<double> wts;
   std::vector<char> isref;
 
+  // trajectory state
   int next_step = 0;
   int head = 0, count = 0;
   std::vector<std::pair<int, int>> log_sites;
   featfix_counters cnt = {0, 0, 0, 0};
   std::vector<Capture> caps;
 
+  // graph of a whole trajectory
+  cudaGraphExec_t gexec = nullptr;
+  bool graph_ok = false;
+  bool capturing = false;
+  long long graph_kernels = 0;
+  std::vector<TimedLaunch> gtimed[NKCLASS];
+
+  // kernel timing
   bool timing[NKCLASS] = {false, false, false, false, false};
   std::vector<TimedLaunch> pending[NKCLASS];
   std::vector<cudaEvent_t> evpool;
@@ -94,6 +131,12 @@ featfix_status fail(featfix_ctx* c, featfix_status s, const std::string& msg) {
       return fail(ctx, FEATFIX_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e__));     \
   } while (0)
 
+#define FF_TRY(call)                          \
+  do {                                        \
+    featfix_status s__ = (call);              \
+    if (s__ != FEATFIX_OK) return s__;        \
+  } while (0)
+
 int n_layers(const featfix_model_desc& d) { return d.arch == FEATFIX_ARCH_MMDIT ? d.n_dual + d.n_single : d.n_dual; }
 
 int patch_vol(const featfix_model_desc& d) { return (d.lat_f > 0 ? d.patch_t : 1) * d.patch * d.patch; }
@@ -112,6 +155,7 @@ std::string check_desc(const featfix_model_desc* d) {
     return "hidden != heads * head_dim";
   if (d->head_dim % 8 || d->head_dim > 128) return "head_dim must be a multiple of 8, <= 128";
   if (d->hidden % 32 || d->mlp <= 0 || d->mlp % 32) return "hidden and mlp must be multiples of 32";
+  if (d->hidden > 4096) return "hidden above 4096";
   if (d->in_ch <= 0 || d->out_ch < d->in_ch) return "bad channel counts";
   if (d->patch <= 0 || d->lat_h % d->patch || d->lat_w % d->patch || d->lat_h <= 0 || d->lat_w <= 0)
     return "latent not divisible by patch";
@@ -119,7 +163,7 @@ std::string check_desc(const featfix_model_desc* d) {
   if (d->txt_tokens < 0) return "bad text length";
   if (d->batch <= 0) return "bad batch";
   const int bm = d->batch * (d->cfg ? 2 : 1);
-  if (bm > 32) return "model batch above 32";
+  if (bm > 64) return "model batch above 64";
   if (d->arch == FEATFIX_ARCH_DIT && d->n_classes <= 0) return "DiT needs classes";
   if (d->rope_dims != 0 && d->rope_dims != 2 && d->rope_dims != 3) return "rope_dims must be 0, 2 or 3";
   if (d->rope_dims == 3 && d->lat_f <= 0) return "3-D rotary needs frames";
@@ -251,7 +295,9 @@ void sampler_coeffs(const featfix_ctx* c, int i, float* c1, float* c2) {
 }
 
 // ---------------------------------------------------------------------------
-// kernel timing
+// kernel timing: CUDA events on the work stream around each launch of a
+// timed kernel class; inside a graph capture the events become external
+// event-record nodes that every replay records again.
 // ---------------------------------------------------------------------------
 cudaEvent_t ev_get(featfix_ctx* c) {
   if (!c->evpool.empty()) {
@@ -270,14 +316,18 @@ struct KTimer {
   double work;
   cudaEvent_t a = nullptr;
   KTimer(featfix_ctx* c_, int k_, double work_) : c(c_), k(k_), work(work_) {
-    if (c->timing[k]) {
-      a = ev_get(c);
-      cudaEventRecord(a, c->st);
-    }
+    if (!c->timing[k]) return;
+    a = ev_get(c);
+    if (c->capturing) cudaEventRecordWithFlags(a, c->st, cudaEventRecordExternal);
+    else cudaEventRecord(a, c->st);
   }
   ~KTimer() {
-    if (a) {
-      cudaEvent_t b = ev_get(c);
+    if (!a) return;
+    cudaEvent_t b = ev_get(c);
+    if (c->capturing) {
+      cudaEventRecordWithFlags(b, c->st, cudaEventRecordExternal);
+      c->gtimed[k].push_back({a, b, work});
+    } else {
       cudaEventRecord(b, c->st);
       c->pending[k].push_back({a, b, work});
     }
@@ -300,13 +350,37 @@ void timing_drain(featfix_ctx* c) {
   }
 }
 
+// After a replay (stream synchronised): the graph's events hold that replay's times.
+void timing_take_graph(featfix_ctx* c) {
+  for (int k = 0; k < NKCLASS; ++k) {
+    if (!c->timing[k]) continue;
+    for (auto& t : c->gtimed[k]) {
+      float ms = 0.f;
+      if (cudaEventElapsedTime(&ms, t.a, t.b) == cudaSuccess) {
+        c->tms[k] += ms;
+        c->twork[k] += t.work;
+        c->tcount[k] += 1;
+      }
+    }
+  }
+}
+
+void graph_reset(featfix_ctx* c) {
+  if (c->gexec) cudaGraphExecDestroy(c->gexec);
+  c->gexec = nullptr;
+  c->graph_ok = false;
+  for (int k = 0; k < NKCLASS; ++k) {
+    for (auto& t : c->gtimed[k]) {
+      c->evpool.push_back(t.a);
+      c->evpool.push_back(t.b);
+    }
+    c->gtimed[k].clear();
+  }
+}
+
 // ---------------------------------------------------------------------------
 // building blocks
 // ---------------------------------------------------------------------------
-template <class T>
-T* at(void* base, long long elems, int es) {
-  return reinterpret_cast<T*>(reinterpret_cast<char*>(base) + elems * es);
-}
 void* off(void* base, long long elems, int es) { return reinterpret_cast<char*>(base) + elems * es; }
 const void* coff(const void* base, long long elems, int es) { return reinterpret_cast<const char*>(base) + elems * es; }
 
@@ -332,39 +406,47 @@ cudaError_t run_attention(featfix_ctx* c, const void* q, const void* k, const vo
   return attention(c->dt, a, c->st);
 }
 
-cudaError_t modvec(featfix_ctx* c, int widx, int chunks, float* out) {
-  KTimer tm(c, FEATFIX_KCLASS_OTHER, 0);
-  return launch_linear_small(c->dt, c->csilu, c->Bm, c->C, c->w[widx], c->w[widx + 1], chunks * c->C, out,
-                             chunks * c->C, 0, 0, c->st);
+// Modulation rows of (step i, block l, stream s): [Bm, chunks*C] at `stride`.
+struct Mod {
+  const float* p;
+  int stride;
+  const float* chunk(int j, int C) const { return p + (size_t)j * C; }
+};
+
+Mod block_mod(featfix_ctx* c, int i, int l, int s) {
+  const int rb = c->mod_row_override >= 0 ? c->mod_row_override : c->need_row[i];
+  return {c->bmodtab + (size_t)rb * c->Bm * c->Nblk + c->moff[2 * l + s], (int)c->Nblk};
 }
 
-cudaError_t ln_mod(featfix_ctx* c, const void* x, void* out, long long rows, const float* mod, int shift_chunk,
-                   int scale_chunk, int stride_chunks, int seg_split, int rpb0, int rpb1) {
+Mod final_mod(featfix_ctx* c, int i) { return {c->fmodtab + (size_t)i * c->Bm * 2 * c->C, 2 * c->C}; }
+
+cudaError_t ln_mod(featfix_ctx* c, const void* x, void* out, long long rows, const Mod& m, int shift_chunk,
+                   int scale_chunk, int seg_split, int rpb0, int rpb1) {
   KTimer tm(c, FEATFIX_KCLASS_OTHER, 0);
-  return launch_ln_mod(c->dt, x, out, rows, c->C, mod + shift_chunk * c->C, mod + scale_chunk * c->C,
-                       stride_chunks * c->C, seg_split, rpb0, rpb1, c->st);
+  return launch_ln_mod(c->dt, x, out, rows, c->C, m.chunk(shift_chunk, c->C), m.chunk(scale_chunk, c->C), m.stride,
+                       seg_split, rpb0, rpb1, c->st);
 }
 
 // Exact DiT block B_l (Eq. 1): u -> out, optional history increment out - u.
-featfix_status block_dit(featfix_ctx* ctx, int l, const void* u, void* out, void* hist) {
+featfix_status block_dit(featfix_ctx* ctx, int i, int l, const void* u, void* out, void* hist) {
   const int C = ctx->C, M = ctx->M, es = ctx->es;
   const long long T = ctx->T;
   const int wb = 11 + 10 * l;
   const auto& W = ctx->w;
-  FF_CK(modvec(ctx, wb, 6, ctx->mod_a));
-  FF_CK(ln_mod(ctx, u, ctx->xm, T, ctx->mod_a, 0, 1, 6, 0, 1, ctx->Ni));
+  const Mod m = block_mod(ctx, i, l, 0);
+  FF_CK(ln_mod(ctx, u, ctx->xm, T, m, 0, 1, 0, 1, ctx->Ni));
   FF_CK(dense(ctx, (int)T, 3 * C, C, ctx->xm, C, W[wb + 2], epi(ctx->qkv, 3 * C, W[wb + 3])));
   FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, es), off(ctx->qkv, 2 * C, es), 3 * C, ctx->att, C));
   EpiArgs e = epi(ctx->u1, C, W[wb + 5]);
-  e.gate = ctx->mod_a + 2 * C; e.gate_stride = 6 * C; e.rpb1 = ctx->Ni;
+  e.gate = m.chunk(2, C); e.gate_stride = m.stride; e.rpb1 = ctx->Ni;
   e.resid = u; e.ld_resid = C;
   FF_CK(dense(ctx, (int)T, C, C, ctx->att, C, W[wb + 4], e));
-  FF_CK(ln_mod(ctx, ctx->u1, ctx->xm, T, ctx->mod_a, 3, 4, 6, 0, 1, ctx->Ni));
+  FF_CK(ln_mod(ctx, ctx->u1, ctx->xm, T, m, 3, 4, 0, 1, ctx->Ni));
   EpiArgs e1 = epi(ctx->big, M, W[wb + 7]);
   e1.act = 1;
   FF_CK(dense(ctx, (int)T, M, C, ctx->xm, C, W[wb + 6], e1));
   EpiArgs e2 = epi(out, C, W[wb + 9]);
-  e2.gate = ctx->mod_a + 5 * C; e2.gate_stride = 6 * C; e2.rpb1 = ctx->Ni;
+  e2.gate = m.chunk(5, C); e2.gate_stride = m.stride; e2.rpb1 = ctx->Ni;
   e2.resid = ctx->u1; e2.ld_resid = C;
   if (hist) { e2.hist_base = u; e2.hist_out = hist; }
   FF_CK(dense(ctx, (int)T, C, M, ctx->big, M, W[wb + 8], e2));
@@ -373,20 +455,17 @@ featfix_status block_dit(featfix_ctx* ctx, int l, const void* u, void* out, void
 
 // Exact MMDiT two-stream block: per-stream modulation and projections,
 // joint attention.  Text rows [0, Bm*Nt), image rows after.
-featfix_status block_dual(featfix_ctx* ctx, int l, const void* u, void* out, void* hist) {
+featfix_status block_dual(featfix_ctx* ctx, int i, int l, const void* u, void* out, void* hist) {
   const int C = ctx->C, M = ctx->M, es = ctx->es;
   const int wb = 10 + 20 * l;
   const auto& W = ctx->w;
   const long long rt = (long long)ctx->Bm * ctx->Nt, ri = (long long)ctx->Bm * ctx->Ni;
-  float* mi = ctx->mod_a;
-  float* mt = ctx->mod_b;
-  FF_CK(modvec(ctx, wb, 6, mi));
-  if (rt) FF_CK(modvec(ctx, wb + 2, 6, mt));
+  const Mod mi = block_mod(ctx, i, l, 0), mt = block_mod(ctx, i, l, 1);
   // stream s: 0 text, 1 image
   for (int s = 0; s < 2; ++s) {
     const long long r0 = s == 0 ? 0 : rt, rows = s == 0 ? rt : ri;
     if (!rows) continue;
-    FF_CK(ln_mod(ctx, coff(u, r0 * C, es), off(ctx->xm, r0 * C, es), rows, s ? mi : mt, 0, 1, 6, 0, 1,
+    FF_CK(ln_mod(ctx, coff(u, r0 * C, es), off(ctx->xm, r0 * C, es), rows, s ? mi : mt, 0, 1, 0, 1,
                  s ? ctx->Ni : ctx->Nt));
     const int wq = s ? wb + 4 : wb + 6;
     EpiArgs e = epi(off(ctx->qkv, r0 * 3 * C, es), 3 * C, W[wq + 1]);
@@ -399,20 +478,20 @@ featfix_status block_dual(featfix_ctx* ctx, int l, const void* u, void* out, voi
   for (int s = 0; s < 2; ++s) {
     const long long r0 = s == 0 ? 0 : rt, rows = s == 0 ? rt : ri;
     if (!rows) continue;
-    float* m = s ? mi : mt;
+    const Mod& m = s ? mi : mt;
     const int rpb = s ? ctx->Ni : ctx->Nt;
     const int wp = s ? wb + 8 : wb + 10;
     EpiArgs e = epi(off(ctx->u1, r0 * C, es), C, W[wp + 1]);
-    e.gate = m + 2 * C; e.gate_stride = 6 * C; e.rpb1 = rpb;
+    e.gate = m.chunk(2, C); e.gate_stride = m.stride; e.rpb1 = rpb;
     e.resid = coff(u, r0 * C, es); e.ld_resid = C;
     FF_CK(dense(ctx, (int)rows, C, C, off(ctx->att, r0 * C, es), C, W[wp], e));
-    FF_CK(ln_mod(ctx, off(ctx->u1, r0 * C, es), off(ctx->xm, r0 * C, es), rows, m, 3, 4, 6, 0, 1, rpb));
+    FF_CK(ln_mod(ctx, off(ctx->u1, r0 * C, es), off(ctx->xm, r0 * C, es), rows, m, 3, 4, 0, 1, rpb));
     const int wf = s ? wb + 12 : wb + 16;
     EpiArgs e1 = epi(off(ctx->big, r0 * M, es), M, W[wf + 1]);
     e1.act = 1;
     FF_CK(dense(ctx, (int)rows, M, C, off(ctx->xm, r0 * C, es), C, W[wf], e1));
     EpiArgs e2 = epi(off(out, r0 * C, es), C, W[wf + 3]);
-    e2.gate = m + 5 * C; e2.gate_stride = 6 * C; e2.rpb1 = rpb;
+    e2.gate = m.chunk(5, C); e2.gate_stride = m.stride; e2.rpb1 = rpb;
     e2.resid = off(ctx->u1, r0 * C, es); e2.ld_resid = C;
     if (hist) { e2.hist_base = coff(u, r0 * C, es); e2.hist_out = off(hist, r0 * C, es); }
     FF_CK(dense(ctx, (int)rows, C, M, off(ctx->big, r0 * M, es), M, W[wf + 2], e2));
@@ -422,14 +501,15 @@ featfix_status block_dual(featfix_ctx* ctx, int l, const void* u, void* out, voi
 
 // Exact MMDiT single-stream block: linear1 -> [q k v | GELU(mlp)] (the MLP
 // half written next to the attention output), joint attention, linear2.
-featfix_status block_single(featfix_ctx* ctx, int l, const void* u, void* out, void* hist) {
+featfix_status block_single(featfix_ctx* ctx, int i, int l, const void* u, void* out, void* hist) {
   const int C = ctx->C, M = ctx->M;
   const int j = l - ctx->d.n_dual;
   const int wb = 10 + 20 * ctx->d.n_dual + 6 * j;
   const auto& W = ctx->w;
   const long long T = ctx->T, rt = (long long)ctx->Bm * ctx->Nt;
-  FF_CK(modvec(ctx, wb, 3, ctx->mod_a));
-  FF_CK(ln_mod(ctx, u, ctx->xm, T, ctx->mod_a, 0, 1, 3, (int)rt, ctx->Nt > 0 ? ctx->Nt : 1, ctx->Ni));
+  const Mod m = block_mod(ctx, i, l, 0);
+  const int rpb0 = ctx->Nt > 0 ? ctx->Nt : 1;
+  FF_CK(ln_mod(ctx, u, ctx->xm, T, m, 0, 1, (int)rt, rpb0, ctx->Ni));
   EpiArgs e = epi(ctx->qkv, 3 * C, W[wb + 3]);
   e.split_col = 3 * C;
   e.out2 = off(ctx->big, C, ctx->es);
@@ -442,30 +522,63 @@ featfix_status block_single(featfix_ctx* ctx, int l, const void* u, void* out, v
   FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, ctx->es), off(ctx->qkv, 2 * C, ctx->es), 3 * C, ctx->big,
                       C + M));
   EpiArgs e2 = epi(out, C, W[wb + 5]);
-  e2.gate = ctx->mod_a + 2 * C; e2.gate_stride = 3 * C;
-  e2.seg_split = (int)rt; e2.rpb0 = ctx->Nt > 0 ? ctx->Nt : 1; e2.rpb1 = ctx->Ni;
+  e2.gate = m.chunk(2, C); e2.gate_stride = m.stride;
+  e2.seg_split = (int)rt; e2.rpb0 = rpb0; e2.rpb1 = ctx->Ni;
   e2.resid = u; e2.ld_resid = C;
   if (hist) { e2.hist_base = u; e2.hist_out = hist; }
   FF_CK(dense(ctx, (int)T, C, C + M, ctx->big, C + M, W[wb + 4], e2));
   return FEATFIX_OK;
 }
 
-featfix_status exact_block(featfix_ctx* ctx, int l, const void* u, void* out, void* hist) {
-  if (ctx->d.arch == FEATFIX_ARCH_DIT) return block_dit(ctx, l, u, out, hist);
-  if (l < ctx->d.n_dual) return block_dual(ctx, l, u, out, hist);
-  return block_single(ctx, l, u, out, hist);
+featfix_status exact_block(featfix_ctx* ctx, int i, int l, const void* u, void* out, void* hist) {
+  if (ctx->d.arch == FEATFIX_ARCH_DIT) return block_dit(ctx, i, l, u, out, hist);
+  if (l < ctx->d.n_dual) return block_dual(ctx, i, l, u, out, hist);
+  return block_single(ctx, i, l, u, out, hist);
 }
 
-// c = MLP(sinusoid(t)) (+ label embedding), SiLU(c) for the modulations.
-featfix_status conditioning(featfix_ctx* ctx, double t, const void* cond) {
-  KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+// Conditioning and every adaLN modulation vector of steps [lo, hi):
+// c = MLP(sinusoid(t)) (+ label embedding), then SiLU(c) times the
+// concatenated modulation weights of all blocks (one GEMM) and of the final
+// layer (one GEMM).  Only c depends on the step, so a whole trajectory's
+// modulations are two tensor-core GEMMs.
+featfix_status compute_mods(featfix_ctx* ctx, const void* cond, int lo, int hi) {
+  const int S = hi - lo, C = ctx->C, Bm = ctx->Bm, es = ctx->es;
   const auto& W = ctx->w;
-  FF_CK(launch_sinusoid((float)t, ctx->sinus, 256, ctx->st));
-  FF_CK(launch_linear_small(ctx->dt, ctx->sinus, 1, 256, W[0], W[1], ctx->C, ctx->thid, ctx->C, 0, 1, ctx->st));
-  FF_CK(launch_linear_small(ctx->dt, ctx->thid, 1, ctx->C, W[2], W[3], ctx->C, ctx->temb, ctx->C, 0, 0, ctx->st));
   const bool dit = ctx->d.arch == FEATFIX_ARCH_DIT;
-  FF_CK(launch_cond_finish(ctx->dt, ctx->temb, dit ? W[4] : nullptr, dit ? (const int*)cond : nullptr, ctx->Bm,
-                           ctx->C, ctx->cvec, ctx->csilu, ctx->st));
+  const int wfin = dit ? 7 : 6;
+  {
+    KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+    FF_CK(launch_sinusoid_table(ctx->dt, ctx->d_times + lo, S, off(ctx->sin_tab, (long long)lo * 256, es), ctx->st));
+  }
+  EpiArgs e1 = epi(off(ctx->thid_tab, (long long)lo * C, es), C, W[1]);
+  e1.act = 2;
+  FF_CK(dense(ctx, S, C, 256, off(ctx->sin_tab, (long long)lo * 256, es), 256, W[0], e1));
+  EpiArgs e2 = epi(ctx->temb_tab + (size_t)lo * C, C, W[3]);
+  e2.out_f32 = 1;
+  FF_CK(dense(ctx, S, C, C, off(ctx->thid_tab, (long long)lo * C, es), C, W[2], e2));
+  // row block of the first step in range that has exact blocks, and how many do
+  int rb0 = -1, nneed = 0;
+  for (int i = lo; i < hi; ++i)
+    if (ctx->need_row[i] >= 0) {
+      if (rb0 < 0) rb0 = ctx->need_row[i];
+      ++nneed;
+    }
+  const bool gather = S > 1;
+  {
+    KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+    FF_CK(launch_cond_table(ctx->dt, ctx->temb_tab + (size_t)lo * C, dit ? W[4] : nullptr,
+                            dit ? (const int*)cond : nullptr, S, Bm, C, gather ? ctx->d_need + lo : nullptr,
+                            off(ctx->cs_all, (long long)lo * Bm * C, es), ctx->cs_need, ctx->st));
+  }
+  EpiArgs ef = epi(ctx->fmodtab + (size_t)lo * Bm * 2 * C, 2 * C, W[wfin + 1]);
+  ef.out_f32 = 1;
+  FF_CK(dense(ctx, S * Bm, 2 * C, C, off(ctx->cs_all, (long long)lo * Bm * C, es), C, W[wfin], ef));
+  if (nneed > 0) {
+    const void* A = gather ? off(ctx->cs_need, (long long)rb0 * Bm * C, es) : off(ctx->cs_all, (long long)lo * Bm * C, es);
+    EpiArgs eb = epi(ctx->bmodtab + (size_t)rb0 * Bm * ctx->Nblk, (int)ctx->Nblk, ctx->bmod);
+    eb.out_f32 = 1;
+    FF_CK(dense(ctx, nneed * Bm, (int)ctx->Nblk, C, A, C, ctx->wmod, eb));
+  }
   return FEATFIX_OK;
 }
 
@@ -488,7 +601,8 @@ featfix_status embed(featfix_ctx* ctx, const float* latent, const void* cond, vo
       KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
       FF_CK(launch_convert(ctx->dt, (const float*)cond, x, rt * C, ctx->st));
     }
-    FF_CK(dense(ctx, ctx->Bm * ctx->Ni, C, ctx->fin, ctx->patches, ctx->fin, ctx->w[4], epi(off(x, rt * C, es), C, ctx->w[5])));
+    FF_CK(dense(ctx, ctx->Bm * ctx->Ni, C, ctx->fin, ctx->patches, ctx->fin, ctx->w[4],
+                epi(off(x, rt * C, es), C, ctx->w[5])));
   }
   return FEATFIX_OK;
 }
@@ -497,11 +611,10 @@ featfix_status embed(featfix_ctx* ctx, const float* latent, const void* cond, vo
 featfix_status finish_step(featfix_ctx* ctx, int i, const void* x, float* latent) {
   const auto& d = ctx->d;
   const int C = ctx->C, es = ctx->es;
-  const bool dit = d.arch == FEATFIX_ARCH_DIT;
-  const int wm = dit ? 7 : 6;
+  const int wm = d.arch == FEATFIX_ARCH_DIT ? 7 : 6;
   const long long rt = (long long)ctx->Bm * ctx->Nt, ri = (long long)ctx->Bm * ctx->Ni;
-  FF_CK(modvec(ctx, wm, 2, ctx->mod_b));
-  FF_CK(ln_mod(ctx, coff(x, rt * C, es), ctx->xm, ri, ctx->mod_b, 0, 1, 2, 0, 1, ctx->Ni));
+  const Mod m = final_mod(ctx, i);
+  FF_CK(ln_mod(ctx, coff(x, rt * C, es), ctx->xm, ri, m, 0, 1, 0, 1, ctx->Ni));
   EpiArgs e = epi(ctx->mout, ctx->fout, ctx->w[wm + 3]);
   e.out_f32 = 1;
   FF_CK(dense(ctx, (int)ri, ctx->fout, C, ctx->xm, C, ctx->w[wm + 2], e));
@@ -523,15 +636,120 @@ Hist4 hist_ptrs(featfix_ctx* c, int l, int nt) {
   return h;
 }
 
+// One denoising step (modulations of step i ready): embedding, the L blocks
+// per the plan (exact / draft / paid site), final layer, sampler update.
+featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* cond) {
+  if (i == 0) {
+    ctx->head = ctx->S - 1;
+    ctx->count = 0;
+    ctx->cnt = {0, 0, 0, 0};
+    ctx->log_sites.clear();
+  }
+  const int L = ctx->L;
+  const bool refresh = ctx->isref[i] != 0;
+  const bool vanilla = ctx->mode == FEATFIX_MODE_VANILLA;
+  const size_t bytes = (size_t)ctx->E * ctx->es;
+  void* x = ctx->xa;
+  void* y = ctx->xb;
+  FF_TRY(embed(ctx, latent, cond, x));
+  const int new_slot = (ctx->head + 1) % ctx->S;
+  const int nt = ctx->keff[i] + 1;
+  float wf[4];
+  for (int j = 0; j < 4; ++j) wf[j] = (float)ctx->wts[(size_t)i * 4 + j];
+  for (int l = 0; l < L; ++l) {
+    for (auto& cp : ctx->caps)
+      if (cp.step == i && cp.layer == l && cp.in) FF_CK(cudaMemcpyAsync(cp.in, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
+    const unsigned char kind = ctx->kinds[(size_t)i * L + l];
+    if (kind == FEATFIX_PLAN_EXACT) {
+      void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, new_slot) : nullptr;
+      FF_TRY(exact_block(ctx, i, l, x, y, hist));
+      std::swap(x, y);
+    } else if (kind == FEATFIX_PLAN_DRAFT) {
+      KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
+      FF_CK(launch_draft(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
+    } else {
+      FF_TRY(exact_block(ctx, i, l, x, y, nullptr));
+      ctx->cnt.paid_checks++;
+      if (ctx->mode != FEATFIX_MODE_EXACT_ONLY) {
+        const int slot = (int)ctx->log_sites.size();
+        if (slot >= ctx->max_logs) return fail(ctx, FEATFIX_ERR_STATE, "log overflow");
+        const int wr = ctx->mode == FEATFIX_MODE_VERIFY ? 1 : 0;
+        KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 2 + wr) * bytes);
+        FF_CK(launch_verify(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, y, ctx->E, wr, ctx->dsums + 4 * slot, ctx->vws,
+                            ctx->st));
+        ctx->log_sites.push_back({i, l});
+      }
+      if (ctx->mode != FEATFIX_MODE_VERIFY) {
+        std::swap(x, y);
+        ctx->cnt.forwarded++;
+      }
+    }
+    for (auto& cp : ctx->caps)
+      if (cp.step == i && cp.layer == l && cp.out) FF_CK(cudaMemcpyAsync(cp.out, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
+  }
+  if (refresh && !vanilla) {
+    ctx->head = new_slot;
+    ctx->count = std::min(ctx->count + 1, ctx->S);
+  }
+  if (refresh || vanilla) ctx->cnt.refresh_steps++;
+  FF_TRY(finish_step(ctx, i, x, latent));
+  ctx->cnt.steps_done = i + 1;
+  ctx->next_step = i + 1;
+  return FEATFIX_OK;
+}
+
+// The whole trajectory on the fixed input buffers g_lat / g_cond.
+featfix_status trajectory(featfix_ctx* ctx) {
+  FF_TRY(compute_mods(ctx, ctx->g_cond, 0, ctx->steps));
+  for (int i = 0; i < ctx->steps; ++i) FF_TRY(step_body(ctx, ctx->g_lat, i, ctx->g_cond));
+  return FEATFIX_OK;
+}
+
+// Capture trajectory() into a graph on the private stream.  The host-side
+// trajectory state (history ring position, counters, log slots) advances
+// during the capture exactly as in a run from step 0, and every replay
+// repeats that run, so the state stays valid after each replay.
+featfix_status build_graph(featfix_ctx* ctx) {
+  graph_reset(ctx);
+  FF_CK(cudaStreamBeginCapture(ctx->cap_st, cudaStreamCaptureModeRelaxed));
+  ctx->st = ctx->cap_st;
+  ctx->capturing = true;
+  const long long k0 = launches_total();
+  const featfix_status s = trajectory(ctx);
+  ctx->capturing = false;
+  ctx->st = ctx->user_st;
+  cudaGraph_t g = nullptr;
+  const cudaError_t e = cudaStreamEndCapture(ctx->cap_st, &g);
+  ctx->graph_kernels = launches_total() - k0;
+  count_launches(-ctx->graph_kernels);  // capturing launched nothing; replays are counted
+  if (s != FEATFIX_OK) {
+    if (g) cudaGraphDestroy(g);
+    graph_reset(ctx);
+    return s;
+  }
+  if (e != cudaSuccess) return fail(ctx, FEATFIX_ERR_CUDA, std::string("graph capture: ") + cudaGetErrorString(e));
+  const cudaError_t e2 = cudaGraphInstantiate(&ctx->gexec, g, 0);
+  cudaGraphDestroy(g);
+  if (e2 != cudaSuccess) {
+    ctx->gexec = nullptr;
+    return fail(ctx, FEATFIX_ERR_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(e2));
+  }
+  ctx->graph_ok = true;
+  return FEATFIX_OK;
+}
+
 void free_all(featfix_ctx* c) {
-  void* bufs[] = {c->xa, c->xb, c->xm, c->qkv, c->att, c->u1, c->big, c->patches, c->pos, c->mod_a, c->mod_b,
-                  c->cvec, c->csilu, c->sinus, c->thid, c->temb, c->mout, c->rope, c->ring, c->dsums, c->vws,
+  graph_reset(c);
+  void* bufs[] = {c->xa, c->xb, c->xm, c->qkv, c->att, c->u1, c->big, c->patches, c->pos, c->mout, c->rope,
+                  c->ring, c->wmod, c->bmod, c->d_times, c->d_need, c->sin_tab, c->thid_tab, c->temb_tab,
+                  c->cs_all, c->cs_need, c->bmodtab, c->fmodtab, c->dsums, c->vws, c->g_lat, c->g_cond,
                   c->h_latent, c->h_cond};
   for (void* p : bufs)
     if (p) cudaFree(p);
   for (int k = 0; k < NKCLASS; ++k)
     for (auto& t : c->pending[k]) { cudaEventDestroy(t.a); cudaEventDestroy(t.b); }
   for (auto e : c->evpool) cudaEventDestroy(e);
+  if (c->cap_st) cudaStreamDestroy(c->cap_st);
 }
 
 featfix_status alloc(featfix_ctx* c, void** p, size_t bytes) {
@@ -541,6 +759,11 @@ featfix_status alloc(featfix_ctx* c, void** p, size_t bytes) {
     return fail(c, FEATFIX_ERR_OOM, "device allocation of " + std::to_string(bytes) + " bytes failed");
   }
   return FEATFIX_OK;
+}
+
+void free_ptr(void** p) {
+  if (*p) cudaFree(*p);
+  *p = nullptr;
 }
 
 // (cos, sin) of every image token / rotary pair: axis widths d/2,d/2 (2-D)
@@ -569,6 +792,115 @@ std::vector<float2> rope_table_host(const featfix_model_desc& d, int hd) {
     }
   }
   return tab;
+}
+
+// Block modulation weights gathered into one [Nblk, C] matrix (and bias);
+// the caller's tensors are copied once here.
+featfix_status gather_mod_weights(featfix_ctx* ctx) {
+  const auto& d = ctx->d;
+  const int C = ctx->C, es = ctx->es;
+  std::vector<std::pair<int, int>> parts;  // (weight index, rows)
+  ctx->moff.assign(2 * (size_t)ctx->L, 0);
+  long long col = 0;
+  for (int l = 0; l < ctx->L; ++l) {
+    if (d.arch == FEATFIX_ARCH_DIT) {
+      ctx->moff[2 * l] = col;
+      parts.push_back({11 + 10 * l, 6 * C});
+      col += 6 * C;
+    } else if (l < d.n_dual) {
+      ctx->moff[2 * l] = col;
+      parts.push_back({10 + 20 * l, 6 * C});
+      col += 6 * C;
+      ctx->moff[2 * l + 1] = col;
+      parts.push_back({10 + 20 * l + 2, 6 * C});
+      col += 6 * C;
+    } else {
+      ctx->moff[2 * l] = col;
+      parts.push_back({10 + 20 * d.n_dual + 6 * (l - d.n_dual), 3 * C});
+      col += 3 * C;
+    }
+  }
+  ctx->Nblk = col;
+  FF_TRY(alloc(ctx, &ctx->wmod, (size_t)col * C * es));
+  FF_TRY(alloc(ctx, &ctx->bmod, (size_t)col * es));
+  long long r = 0;
+  for (auto& p : parts) {
+    FF_CK(cudaMemcpyAsync(off(ctx->wmod, r * C, es), ctx->w[p.first], (size_t)p.second * C * es,
+                          cudaMemcpyDeviceToDevice, ctx->user_st));
+    FF_CK(cudaMemcpyAsync(off(ctx->bmod, r, es), ctx->w[p.first + 1], (size_t)p.second * es,
+                          cudaMemcpyDeviceToDevice, ctx->user_st));
+    r += p.second;
+  }
+  return FEATFIX_OK;
+}
+
+featfix_status create_impl(featfix_ctx* ctx) {
+  const featfix_model_desc& d = ctx->d;
+  const int es = ctx->es;
+  const long long T = ctx->T, C = ctx->C, M = ctx->M;
+  FF_CK(cudaStreamCreateWithFlags(&ctx->cap_st, cudaStreamNonBlocking));
+  FF_TRY(alloc(ctx, &ctx->xa, T * C * es));
+  FF_TRY(alloc(ctx, &ctx->xb, T * C * es));
+  FF_TRY(alloc(ctx, &ctx->xm, T * C * es));
+  FF_TRY(alloc(ctx, &ctx->qkv, T * 3 * C * es));
+  FF_TRY(alloc(ctx, &ctx->att, T * C * es));
+  FF_TRY(alloc(ctx, &ctx->u1, T * C * es));
+  FF_TRY(alloc(ctx, &ctx->big, T * (C + M) * es));
+  FF_TRY(alloc(ctx, &ctx->patches, (size_t)ctx->Bm * ctx->Ni * ctx->fin * es));
+  FF_TRY(alloc(ctx, (void**)&ctx->mout, (size_t)ctx->Bm * ctx->Ni * ctx->fout * 4));
+  ctx->lat_elems = (long long)d.batch * d.in_ch * (d.lat_f > 0 ? d.lat_f : 1) * d.lat_h * d.lat_w;
+  ctx->cond_bytes = d.arch == FEATFIX_ARCH_DIT ? (size_t)ctx->Bm * sizeof(int)
+                                              : (size_t)ctx->Bm * ctx->Nt * ctx->C * sizeof(float);
+  FF_TRY(alloc(ctx, (void**)&ctx->g_lat, (size_t)ctx->lat_elems * 4));
+  FF_TRY(alloc(ctx, &ctx->g_cond, ctx->cond_bytes));
+  if (d.arch == FEATFIX_ARCH_DIT) {
+    FF_TRY(alloc(ctx, &ctx->pos, (size_t)ctx->Bm * ctx->Ni * C * es));
+    FF_CK(launch_pos2d(ctx->dt, ctx->pos, ctx->Bm, ctx->gh, ctx->gw, ctx->C, ctx->user_st));
+  }
+  if (d.arch == FEATFIX_ARCH_MMDIT && d.rope_dims) {
+    FF_TRY(alloc(ctx, (void**)&ctx->rope, (size_t)ctx->Ni * (ctx->hd / 2) * sizeof(float2)));
+    std::vector<float2> tab = rope_table_host(d, ctx->hd);
+    FF_CK(cudaMemcpyAsync(ctx->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice, ctx->user_st));
+    FF_CK(cudaStreamSynchronize(ctx->user_st));
+  }
+  FF_TRY(gather_mod_weights(ctx));
+  FF_CK(cudaStreamSynchronize(ctx->user_st));
+  return FEATFIX_OK;
+}
+
+// Per-schedule device state: history ring, modulation tables, logs.
+featfix_status schedule_buffers(featfix_ctx* ctx, int steps, int K, int mode, int n_sites) {
+  const int es = ctx->es, C = ctx->C, Bm = ctx->Bm;
+  const int S = K + 1;
+  if (ctx->ring && ctx->S != S) free_ptr(&ctx->ring);
+  if (!ctx->ring && mode != FEATFIX_MODE_VANILLA) FF_TRY(alloc(ctx, &ctx->ring, (size_t)ctx->L * S * ctx->E * es));
+  ctx->S = S;
+  const int nlog = std::max(n_sites, 1);
+  if (nlog > ctx->max_logs) {
+    free_ptr((void**)&ctx->dsums);
+    FF_TRY(alloc(ctx, (void**)&ctx->dsums, (size_t)nlog * 4 * sizeof(double)));
+    ctx->max_logs = nlog;
+  }
+  const size_t need = verify_workspace_bytes(ctx->E);
+  if (need > ctx->vws_bytes) {
+    free_ptr(&ctx->vws);
+    FF_TRY(alloc(ctx, &ctx->vws, need));
+    ctx->vws_bytes = need;
+  }
+  void** tabs[] = {(void**)&ctx->d_times, (void**)&ctx->d_need, &ctx->sin_tab, &ctx->thid_tab, (void**)&ctx->temb_tab,
+                   &ctx->cs_all, &ctx->cs_need, (void**)&ctx->bmodtab, (void**)&ctx->fmodtab};
+  for (void** p : tabs) free_ptr(p);
+  const int nn = std::max(ctx->n_need, 1);
+  FF_TRY(alloc(ctx, (void**)&ctx->d_times, (size_t)steps * 4));
+  FF_TRY(alloc(ctx, (void**)&ctx->d_need, (size_t)steps * 4));
+  FF_TRY(alloc(ctx, &ctx->sin_tab, (size_t)steps * 256 * es));
+  FF_TRY(alloc(ctx, &ctx->thid_tab, (size_t)steps * C * es));
+  FF_TRY(alloc(ctx, (void**)&ctx->temb_tab, (size_t)steps * C * 4));
+  FF_TRY(alloc(ctx, &ctx->cs_all, (size_t)steps * Bm * C * es));
+  FF_TRY(alloc(ctx, &ctx->cs_need, (size_t)nn * Bm * C * es));
+  FF_TRY(alloc(ctx, (void**)&ctx->bmodtab, (size_t)(nn + 1) * Bm * ctx->Nblk * 4));
+  FF_TRY(alloc(ctx, (void**)&ctx->fmodtab, (size_t)steps * Bm * 2 * C * 4));
+  return FEATFIX_OK;
 }
 
 }  // namespace
@@ -630,8 +962,7 @@ featfix_status featfix_create(const featfix_model_desc* desc, const void* const*
                               void* cuda_stream, featfix_ctx** out) {
   if (!out) return FEATFIX_ERR_INVALID_ARG;
   *out = nullptr;
-  const std::string why = check_desc(desc);
-  if (!why.empty()) return FEATFIX_ERR_INVALID_ARG;
+  if (!check_desc(desc).empty()) return FEATFIX_ERR_INVALID_ARG;
   const int nw = featfix_weight_count(desc);
   if (!dev_weights || n_weights != nw) return FEATFIX_ERR_INVALID_ARG;
   for (int k = 0; k < nw; ++k)
@@ -660,46 +991,9 @@ featfix_status featfix_create(const featfix_model_desc* desc, const void* const*
   ctx->gh = d.lat_h / d.patch;
   ctx->gw = d.lat_w / d.patch;
   ctx->w.assign(dev_weights, dev_weights + nw);
-  ctx->st = reinterpret_cast<cudaStream_t>(cuda_stream);
-
-  const int es = ctx->es;
-  const long long T = ctx->T, C = ctx->C, M = ctx->M;
-  featfix_status s = FEATFIX_OK;
-  auto A = [&](void** p, size_t bytes) {
-    if (s == FEATFIX_OK) s = alloc(ctx, p, bytes);
-  };
-  A(&ctx->xa, T * C * es);
-  A(&ctx->xb, T * C * es);
-  A(&ctx->xm, T * C * es);
-  A(&ctx->qkv, T * 3 * C * es);
-  A(&ctx->att, T * C * es);
-  A(&ctx->u1, T * C * es);
-  A(&ctx->big, T * (C + M) * es);
-  A(&ctx->patches, (size_t)ctx->Bm * ctx->Ni * ctx->fin * es);
-  A((void**)&ctx->mod_a, (size_t)ctx->Bm * 6 * C * 4);
-  A((void**)&ctx->mod_b, (size_t)ctx->Bm * 6 * C * 4);
-  A((void**)&ctx->cvec, (size_t)ctx->Bm * C * 4);
-  A((void**)&ctx->csilu, (size_t)ctx->Bm * C * 4);
-  A((void**)&ctx->sinus, 256 * 4);
-  A((void**)&ctx->thid, C * 4);
-  A((void**)&ctx->temb, C * 4);
-  A((void**)&ctx->mout, (size_t)ctx->Bm * ctx->Ni * ctx->fout * 4);
-  if (d.arch == FEATFIX_ARCH_DIT) A(&ctx->pos, (size_t)ctx->Bm * ctx->Ni * C * es);
-  if (d.arch == FEATFIX_ARCH_MMDIT && d.rope_dims) A((void**)&ctx->rope, (size_t)ctx->Ni * (ctx->hd / 2) * sizeof(float2));
-  if (s != FEATFIX_OK) {
-    free_all(ctx);
-    delete ctx;
-    return s;
-  }
-  if (d.arch == FEATFIX_ARCH_DIT && launch_pos2d(ctx->dt, ctx->pos, ctx->Bm, ctx->gh, ctx->gw, ctx->C, ctx->st) != cudaSuccess)
-    s = FEATFIX_ERR_CUDA;
-  if (ctx->rope) {
-    std::vector<float2> tab = rope_table_host(d, ctx->hd);
-    if (cudaMemcpyAsync(ctx->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice, ctx->st) !=
-            cudaSuccess ||
-        cudaStreamSynchronize(ctx->st) != cudaSuccess)
-      s = FEATFIX_ERR_CUDA;
-  }
+  ctx->user_st = reinterpret_cast<cudaStream_t>(cuda_stream);
+  ctx->st = ctx->user_st;
+  const featfix_status s = create_impl(ctx);
   if (s != FEATFIX_OK) {
     free_all(ctx);
     delete ctx;
@@ -711,7 +1005,7 @@ featfix_status featfix_create(const featfix_model_desc* desc, const void* const*
 
 void featfix_destroy(featfix_ctx* ctx) {
   if (!ctx) return;
-  cudaStreamSynchronize(ctx->st);
+  cudaStreamSynchronize(ctx->user_st);
   free_all(ctx);
   delete ctx;
 }
@@ -729,38 +1023,29 @@ featfix_status featfix_set_schedule(featfix_ctx* ctx, int steps, const int* refr
   if (s != FEATFIX_OK) return fail(ctx, s, err);
   if (ctx->d.sampler == FEATFIX_SAMPLER_DDIM && (1000 % steps != 0))
     return fail(ctx, FEATFIX_ERR_UNSUPPORTED, "DDIM needs steps dividing 1000");
-  cudaStreamSynchronize(ctx->st);
-  const int S = draft_order + 1;
-  if (ctx->ring && ctx->S != S) {
-    cudaFree(ctx->ring);
-    ctx->ring = nullptr;
+  FF_CK(cudaStreamSynchronize(ctx->user_st));
+  graph_reset(ctx);
+  ctx->sched = false;
+  // steps whose blocks need modulation vectors (any exact block or site)
+  std::vector<int> need(steps, -1);
+  int nn = 0;
+  for (int i = 0; i < steps; ++i) {
+    bool any = false;
+    for (int l = 0; l < ctx->L; ++l) any |= kd[(size_t)i * ctx->L + l] != FEATFIX_PLAN_DRAFT;
+    if (any) need[i] = nn++;
   }
-  if (!ctx->ring && mode != FEATFIX_MODE_VANILLA) {
-    s = alloc(ctx, &ctx->ring, (size_t)ctx->L * S * ctx->E * ctx->es);
-    if (s != FEATFIX_OK) return s;
-  }
-  ctx->S = S;
-  const int nlog = std::max(n_sites, 1);
-  if (nlog > ctx->max_logs) {
-    if (ctx->dsums) cudaFree(ctx->dsums);
-    ctx->dsums = nullptr;
-    s = alloc(ctx, (void**)&ctx->dsums, (size_t)nlog * 4 * sizeof(double));
-    if (s != FEATFIX_OK) return s;
-    ctx->max_logs = nlog;
-  }
-  const size_t need = verify_workspace_bytes(ctx->E);
-  if (need > ctx->vws_bytes) {
-    if (ctx->vws) cudaFree(ctx->vws);
-    ctx->vws = nullptr;
-    s = alloc(ctx, &ctx->vws, need);
-    if (s != FEATFIX_OK) return s;
-    ctx->vws_bytes = need;
-  }
+  ctx->n_need = nn;
+  FF_TRY(schedule_buffers(ctx, steps, draft_order, mode, n_sites));
+  ctx->need_row = need;
+  ctx->steps = steps;
+  std::vector<float> times(steps);
+  for (int i = 0; i < steps; ++i) times[i] = (float)model_time(ctx, i);
+  FF_CK(cudaMemcpy(ctx->d_times, times.data(), steps * sizeof(float), cudaMemcpyHostToDevice));
+  FF_CK(cudaMemcpy(ctx->d_need, need.data(), steps * sizeof(int), cudaMemcpyHostToDevice));
   ctx->kinds.swap(kd);
   ctx->keff.swap(ke);
   ctx->wts.swap(wt);
   ctx->isref.swap(isref);
-  ctx->steps = steps;
   ctx->K = draft_order;
   ctx->mode = mode;
   ctx->flags = flags;
@@ -786,69 +1071,8 @@ featfix_status featfix_step(featfix_ctx* ctx, float* latent, int i, const void* 
   if (!ctx->sched) return fail(ctx, FEATFIX_ERR_STATE, "featfix_set_schedule first");
   if (i != 0 && i != ctx->next_step) return fail(ctx, FEATFIX_ERR_STATE, "step out of order");
   if (i >= ctx->steps) return fail(ctx, FEATFIX_ERR_STATE, "step beyond the schedule");
-  if (i == 0) {
-    ctx->head = ctx->S - 1;
-    ctx->count = 0;
-    ctx->cnt = {0, 0, 0, 0};
-    ctx->log_sites.clear();
-  }
-  const int L = ctx->L;
-  const bool refresh = ctx->isref[i] != 0;
-  const bool vanilla = ctx->mode == FEATFIX_MODE_VANILLA;
-  const size_t bytes = (size_t)ctx->E * ctx->es;
-  featfix_status s = conditioning(ctx, model_time(ctx, i), cond);
-  if (s != FEATFIX_OK) return s;
-  void* x = ctx->xa;
-  void* y = ctx->xb;
-  s = embed(ctx, latent, cond, x);
-  if (s != FEATFIX_OK) return s;
-  const int new_slot = (ctx->head + 1) % ctx->S;
-  const int nt = ctx->keff[i] + 1;
-  float wf[4];
-  for (int j = 0; j < 4; ++j) wf[j] = (float)ctx->wts[(size_t)i * 4 + j];
-  for (int l = 0; l < L; ++l) {
-    for (auto& cp : ctx->caps)
-      if (cp.step == i && cp.layer == l && cp.in) FF_CK(cudaMemcpyAsync(cp.in, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
-    const unsigned char kind = ctx->kinds[(size_t)i * L + l];
-    if (kind == FEATFIX_PLAN_EXACT) {
-      void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, new_slot) : nullptr;
-      s = exact_block(ctx, l, x, y, hist);
-      if (s != FEATFIX_OK) return s;
-      std::swap(x, y);
-    } else if (kind == FEATFIX_PLAN_DRAFT) {
-      KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
-      FF_CK(launch_draft(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
-    } else {
-      s = exact_block(ctx, l, x, y, nullptr);
-      if (s != FEATFIX_OK) return s;
-      ctx->cnt.paid_checks++;
-      if (ctx->mode != FEATFIX_MODE_EXACT_ONLY) {
-        const int slot = (int)ctx->log_sites.size();
-        if (slot >= ctx->max_logs) return fail(ctx, FEATFIX_ERR_STATE, "log overflow");
-        const int wr = ctx->mode == FEATFIX_MODE_VERIFY ? 1 : 0;
-        KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 2 + wr) * bytes);
-        FF_CK(launch_verify(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, y, ctx->E, wr, ctx->dsums + 4 * slot, ctx->vws,
-                            ctx->st));
-        ctx->log_sites.push_back({i, l});
-      }
-      if (ctx->mode != FEATFIX_MODE_VERIFY) {
-        std::swap(x, y);
-        ctx->cnt.forwarded++;
-      }
-    }
-    for (auto& cp : ctx->caps)
-      if (cp.step == i && cp.layer == l && cp.out) FF_CK(cudaMemcpyAsync(cp.out, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
-  }
-  if (refresh && !vanilla) {
-    ctx->head = new_slot;
-    ctx->count = std::min(ctx->count + 1, ctx->S);
-  }
-  if (refresh || vanilla) ctx->cnt.refresh_steps++;
-  s = finish_step(ctx, i, x, latent);
-  if (s != FEATFIX_OK) return s;
-  ctx->cnt.steps_done = i + 1;
-  ctx->next_step = i + 1;
-  return FEATFIX_OK;
+  FF_TRY(compute_mods(ctx, cond, i, i + 1));
+  return step_body(ctx, latent, i, cond);
 }
 
 featfix_status featfix_sample(featfix_ctx* ctx, unsigned long long seed, int steps, const void* cond,
@@ -857,15 +1081,20 @@ featfix_status featfix_sample(featfix_ctx* ctx, unsigned long long seed, int ste
   if (!ctx->sched) return fail(ctx, FEATFIX_ERR_STATE, "featfix_set_schedule first");
   if (steps != ctx->steps) return fail(ctx, FEATFIX_ERR_SCHEDULE, "steps differ from the schedule");
   if (!latent_out || !cond) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "null latent or cond");
-  const auto& d = ctx->d;
-  const long long n = (long long)d.batch * d.in_ch * (d.lat_f > 0 ? d.lat_f : 1) * d.lat_h * d.lat_w;
+  FF_CK(cudaMemcpyAsync(ctx->g_cond, cond, ctx->cond_bytes, cudaMemcpyDeviceToDevice, ctx->user_st));
   {
     KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
-    FF_CK(launch_noise(seed, latent_out, n, ctx->st));
+    FF_CK(launch_noise(seed, ctx->g_lat, ctx->lat_elems, ctx->user_st));
   }
-  for (int i = 0; i < steps; ++i) {
-    featfix_status s = featfix_step(ctx, latent_out, i, cond);
-    if (s != FEATFIX_OK) return s;
+  if (!ctx->graph_ok) FF_TRY(build_graph(ctx));
+  FF_CK(cudaGraphLaunch(ctx->gexec, ctx->user_st));
+  count_launches(ctx->graph_kernels);
+  FF_CK(cudaMemcpyAsync(latent_out, ctx->g_lat, (size_t)ctx->lat_elems * 4, cudaMemcpyDeviceToDevice, ctx->user_st));
+  bool timed = false;
+  for (int k = 0; k < NKCLASS; ++k) timed |= ctx->timing[k];
+  if (timed) {
+    FF_CK(cudaStreamSynchronize(ctx->user_st));
+    timing_take_graph(ctx);
   }
   return FEATFIX_OK;
 }
@@ -874,25 +1103,19 @@ featfix_status featfix_sample_host(featfix_ctx* ctx, unsigned long long seed, in
                                    float* latent_out_host) {
   if (!ctx) return FEATFIX_ERR_INVALID_ARG;
   if (!cond_host || !latent_out_host) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "null host buffer");
-  const auto& d = ctx->d;
-  const size_t nlat = (size_t)d.batch * d.in_ch * (d.lat_f > 0 ? d.lat_f : 1) * d.lat_h * d.lat_w;
-  const size_t cbytes = d.arch == FEATFIX_ARCH_DIT ? (size_t)ctx->Bm * sizeof(int)
-                                                    : (size_t)ctx->Bm * ctx->Nt * ctx->C * sizeof(float);
-  featfix_status s = FEATFIX_OK;
-  if (!ctx->h_latent) s = alloc(ctx, (void**)&ctx->h_latent, nlat * sizeof(float));
-  if (s == FEATFIX_OK && !ctx->h_cond) s = alloc(ctx, &ctx->h_cond, cbytes);
-  if (s != FEATFIX_OK) return s;
-  FF_CK(cudaMemcpyAsync(ctx->h_cond, cond_host, cbytes, cudaMemcpyHostToDevice, ctx->st));
-  s = featfix_sample(ctx, seed, steps, ctx->h_cond, ctx->h_latent);
-  if (s != FEATFIX_OK) return s;
-  FF_CK(cudaMemcpyAsync(latent_out_host, ctx->h_latent, nlat * sizeof(float), cudaMemcpyDeviceToHost, ctx->st));
-  FF_CK(cudaStreamSynchronize(ctx->st));
+  if (!ctx->h_latent) FF_TRY(alloc(ctx, (void**)&ctx->h_latent, (size_t)ctx->lat_elems * sizeof(float)));
+  if (!ctx->h_cond) FF_TRY(alloc(ctx, &ctx->h_cond, ctx->cond_bytes));
+  FF_CK(cudaMemcpyAsync(ctx->h_cond, cond_host, ctx->cond_bytes, cudaMemcpyHostToDevice, ctx->user_st));
+  FF_TRY(featfix_sample(ctx, seed, steps, ctx->h_cond, ctx->h_latent));
+  FF_CK(cudaMemcpyAsync(latent_out_host, ctx->h_latent, (size_t)ctx->lat_elems * sizeof(float),
+                        cudaMemcpyDeviceToHost, ctx->user_st));
+  FF_CK(cudaStreamSynchronize(ctx->user_st));
   return FEATFIX_OK;
 }
 
 featfix_status featfix_get_log(featfix_ctx* ctx, featfix_site_log* out, int cap, int* n, featfix_counters* counters) {
   if (!ctx) return FEATFIX_ERR_INVALID_ARG;
-  FF_CK(cudaStreamSynchronize(ctx->st));
+  FF_CK(cudaStreamSynchronize(ctx->user_st));
   const unsigned int wd = gemm_tc_watchdog_take();
   if (wd) return fail(ctx, FEATFIX_ERR_CUDA, "tensor-core GEMM watchdog fired (code " + std::to_string(wd) + ")");
   const int avail = (int)ctx->log_sites.size();
@@ -919,11 +1142,13 @@ featfix_status featfix_debug_capture(featfix_ctx* ctx, int step, int layer, void
   if (!ctx) return FEATFIX_ERR_INVALID_ARG;
   if (step < 0) {
     ctx->caps.clear();
+    graph_reset(ctx);
     return FEATFIX_OK;
   }
   if (layer < 0 || layer >= ctx->L || (!dev_in && !dev_out)) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "bad capture");
-  if (ctx->caps.size() >= 32) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "too many captures");
+  if (ctx->caps.size() >= 64) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "too many captures");
   ctx->caps.push_back({step, layer, dev_in, dev_out});
+  graph_reset(ctx);
   return FEATFIX_OK;
 }
 
@@ -933,15 +1158,24 @@ featfix_status featfix_debug_block(featfix_ctx* ctx, int step, int layer, const 
   if (!ctx->sched) return fail(ctx, FEATFIX_ERR_STATE, "featfix_set_schedule first");
   if (step < 0 || step >= ctx->steps || layer < 0 || layer >= ctx->L || !dev_in || !dev_out || !cond)
     return fail(ctx, FEATFIX_ERR_INVALID_ARG, "bad debug block request");
-  featfix_status s = conditioning(ctx, model_time(ctx, step), cond);
+  // modulations of `step` into the spare row block of the table
+  const int spare = std::max(ctx->n_need, 1);
+  const int saved = ctx->need_row[step];
+  ctx->need_row[step] = spare;
+  featfix_status s = compute_mods(ctx, cond, step, step + 1);
+  ctx->need_row[step] = saved;
   if (s != FEATFIX_OK) return s;
-  return exact_block(ctx, layer, dev_in, dev_out, nullptr);
+  ctx->mod_row_override = spare;
+  s = exact_block(ctx, step, layer, dev_in, dev_out, nullptr);
+  ctx->mod_row_override = -1;
+  return s;
 }
 
 featfix_status featfix_kernel_timing(featfix_ctx* ctx, int kclass, int on) {
   if (!ctx || kclass < 0 || kclass >= NKCLASS) return FEATFIX_ERR_INVALID_ARG;
-  FF_CK(cudaStreamSynchronize(ctx->st));
+  FF_CK(cudaStreamSynchronize(ctx->user_st));
   timing_drain(ctx);
+  if (ctx->timing[kclass] != (on != 0)) graph_reset(ctx);
   ctx->timing[kclass] = on != 0;
   ctx->tms[kclass] = 0;
   ctx->twork[kclass] = 0;
@@ -951,7 +1185,7 @@ featfix_status featfix_kernel_timing(featfix_ctx* ctx, int kclass, int on) {
 
 featfix_status featfix_kernel_time(featfix_ctx* ctx, int kclass, double* ms, long long* launches, double* work) {
   if (!ctx || kclass < 0 || kclass >= NKCLASS) return FEATFIX_ERR_INVALID_ARG;
-  FF_CK(cudaStreamSynchronize(ctx->st));
+  FF_CK(cudaStreamSynchronize(ctx->user_st));
   timing_drain(ctx);
   if (ms) *ms = ctx->tms[kclass];
   if (launches) *launches = ctx->tcount[kclass];

@@ -136,6 +136,7 @@ GEMM_SHAPES = [
     (130, 32, 64),        # final projection width
     (512, 3456, 1152),    # DiT-XL/2 qkv width, several N tiles
     (4096, 1152, 4608),   # DiT-XL/2 fc2, full size
+    (4096, 4608, 1152),   # DiT-XL/2 fc1, full size
 ]
 
 
