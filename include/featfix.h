@@ -70,6 +70,17 @@ enum { FEATFIX_PLAN_EXACT = 0, FEATFIX_PLAN_DRAFT = 1, FEATFIX_PLAN_SITE = 2 };
  * the spacing of the two refreshes it joins) instead of the default
  * derivatives of the polynomial interpolating the last K+1 refreshes.  */
 #define FEATFIX_FLAG_TAYLOR_RECURSIVE 1u
+/* PER_BLOCK_DRAFT forces one draft kernel per block at every drafted step.
+ * By default a drafted step without a FeatFix/Exact-only site is evaluated
+ * in one pass: at a full-refresh step every block is exact and each block's
+ * input is the previous block's output, so the per-block increments
+ * telescope, sum_l R_l = x_L - x_0; the forecast of the whole step is then
+ * x_0 + sum_j w_j (x_L - x_0)_{s_j}, the same value as chaining the L
+ * per-block drafts (up to rounding).  In the Verify arm every drafted step
+ * is evaluated this way (so its forwarded trajectory is the one without
+ * sites) and the paid check runs on a shadow copy that chains the per-block
+ * drafts up to the site.  Steps with a debug capture always run per block. */
+#define FEATFIX_FLAG_PER_BLOCK_DRAFT 2u
 
 /*
  * Model shape (Eq. 1's block B_l and the surrounding sampler).

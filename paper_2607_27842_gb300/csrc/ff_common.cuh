@@ -56,6 +56,14 @@ __device__ __forceinline__ float gelu_tanh(float x) {
   const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
   return 0.5f * x * (1.0f + tanhf(k0 * (x + 0.044715f * x * x * x)));
 }
+// Same GELU through the hardware tanh approximation (tanh.approx.f32, about
+// 2^-11 relative error): for bf16 outputs, whose rounding is 2^-9.
+__device__ __forceinline__ float gelu_tanh_fast(float x) {
+  const float k0 = 0.7978845608028654f;
+  float t;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(k0 * (x + 0.044715f * x * x * x)));
+  return 0.5f * x * (1.0f + t);
+}
 __device__ __forceinline__ float silu(float x) { return x / (1.0f + expf(-x)); }
 
 // ---------------------------------------------------------------------------
@@ -135,7 +143,7 @@ __device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N
   }
   if (e.act == 1 && n0 >= e.act_col0) {
 #pragma unroll
-    for (int j = 0; j < CH; ++j) v[j] = gelu_tanh(v[j]);
+    for (int j = 0; j < CH; ++j) v[j] = sizeof(T) == 2 ? gelu_tanh_fast(v[j]) : gelu_tanh(v[j]);
   } else if (e.act == 2 && n0 >= e.act_col0) {
 #pragma unroll
     for (int j = 0; j < CH; ++j) v[j] = silu(v[j]);
@@ -217,6 +225,7 @@ inline cudaError_t launched() {
 }
 
 cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int nt, long long n, cudaStream_t s);
+cudaError_t launch_diff(DType dt, const void* a, const void* b, void* out, long long n, cudaStream_t s);
 size_t verify_workspace_bytes(long long n);
 cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
                           int write_draft, double* sums, void* ws, cudaStream_t s);

@@ -99,6 +99,37 @@ cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int 
   return dt == F32 ? draft_t<float>(x, h, w, nt, n, s) : draft_t<bf16>(x, h, w, nt, n, s);
 }
 
+// out = a - b elementwise (fp32 arithmetic, rounded to the storage type).
+template <class T>
+__global__ void __launch_bounds__(256) k_diff(const T* __restrict__ a, const T* __restrict__ b, T* __restrict__ out,
+                                              long long n) {
+  constexpr int V = VecN<T>::n;
+  const long long nvec = n / V;
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += stride) {
+    float x[V], y[V];
+    ld16(a + i * V, x);
+    ld16(b + i * V, y);
+#pragma unroll
+    for (int q = 0; q < V; ++q) x[q] -= y[q];
+    st16(out + i * V, x);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < n - nvec * V) {
+    const long long i = nvec * V + threadIdx.x;
+    out[i] = from_f<T>(to_f(a[i]) - to_f(b[i]));
+  }
+}
+
+cudaError_t launch_diff(DType dt, const void* a, const void* b, void* out, long long n, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  if (dt == F32) {
+    k_diff<float><<<stream_grid(n / 4, 256), 256, 0, s>>>((const float*)a, (const float*)b, (float*)out, n);
+  } else {
+    k_diff<bf16><<<stream_grid(n / 8, 256), 256, 0, s>>>((const bf16*)a, (const bf16*)b, (bf16*)out, n);
+  }
+  return launched();
+}
+
 // ---------------------------------------------------------------------------
 // Paid check + forward (Eqs. 3-5), fused so h_f is read once: each thread
 // rebuilds h_d from u and the history exactly as k_draft does, accumulates

@@ -61,12 +61,14 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
 __device__ __forceinline__ void mbar_arrive(uint64_t* b) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(saddr(b)) : "memory");
 }
+// try_wait with a suspend-time hint: the waiting thread sleeps in hardware
+// (up to ~0.1 ms) instead of re-issuing the poll.
 __device__ __forceinline__ bool mbar_try(uint64_t* b, uint32_t parity) {
   uint32_t ok;
   asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}\n"
       : "=r"(ok)
-      : "r"(saddr(b)), "r"(parity)
+      : "r"(saddr(b)), "r"(parity), "r"(100000u)
       : "memory");
   return ok != 0;
 }
@@ -94,6 +96,34 @@ __device__ __forceinline__ void tma_load(const CUtensorMap* tm, uint64_t* bar, v
           saddr(dst)),
       "l"((uint64_t)tm), "r"(x), "r"(y), "r"(saddr(bar))
       : "memory");
+}
+
+// ---- CTA-pair (2-SM) helpers --------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// shared::cluster address of the same object in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t map_to(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr(p)), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// TMA load into this CTA's shared memory that completes on an mbarrier of
+// either CTA of the pair (shared::cluster address).
+__device__ __forceinline__ void tma_load_pair(const CUtensorMap* tm, uint32_t bar_cluster, void* dst, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+      "[%4];" ::"r"(saddr(dst)),
+      "l"((uint64_t)tm), "r"(x), "r"(y), "r"(bar_cluster)
+      : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 
 // Shared-memory matrix descriptor, K-major operand with 128-byte swizzle:
@@ -273,6 +303,182 @@ __global__ void __launch_bounds__(THREADS, 1)
 }
 
 // ---------------------------------------------------------------------------
+// CTA-pair variant: a cluster of 2 CTAs computes a 256 x BN tile with
+// tcgen05.mma.cta_group::2 (M = 256).  Each CTA stages its own 128 rows of A
+// and half (BN/2 rows) of W, so per CTA the shared-memory traffic per FLOP
+// is that of a 128 x 2BN tile.  The even CTA issues the MMAs; its full
+// barriers collect both CTAs' TMA bytes; commits are multicast to both CTAs'
+// empty / accumulator-full barriers; both CTAs' epilogues arrive on the even
+// CTA's accumulator-empty barrier.
+// ---------------------------------------------------------------------------
+template <int BN> struct Cfg2 {
+  static constexpr int HB = BN / 2;
+  static constexpr int STAGES = BN >= 256 ? 6 : 8;
+  static constexpr uint32_t A_BYTES = BM * BK * 2;
+  static constexpr uint32_t B_BYTES = HB * BK * 2;
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + 256;
+  static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                                    ((uint32_t)(256 >> 4) << 24);
+};
+
+__device__ __forceinline__ void umma_pair(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+          d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accum));
+}
+// arrive on the mbarrier at this offset in both CTAs of the pair once the
+// issued MMAs complete
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
+  const uint16_t mask = 3;
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          saddr(bar)),
+      "h"(mask)
+      : "memory");
+}
+
+template <int BN>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+    k_gemm_tc2(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
+               EpiArgs e) {
+  using C = Cfg2<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* tfull = empty + C::STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const int num_m = (M + 2 * BM - 1) / (2 * BM), num_n = (N + BN - 1) / BN;
+  const int num_tiles = num_m * num_n;
+  const int num_kb = (K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 2 * 128);
+    }
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(tmem_slot)),
+                 "r"(C::TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncwarp();
+  cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA use
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
+        const int mb = tile % num_m, nb = tile / num_m;
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % C::STAGES;
+          const uint32_t ph = (it / C::STAGES) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
+          if (leader) mbar_expect_tx(&full[s], 2 * C::STAGE_BYTES);
+          const uint32_t fb = map_to(&full[s], 0);
+          tma_load_pair(&tmA, fb, sA + s * C::A_BYTES, kb * BK, mb * 2 * BM + (int)rank * BM);
+          tma_load_pair(&tmB, fb, sB + s * C::B_BYTES, kb * BK, nb * BN + (int)rank * C::HB);
+        }
+      }
+      if (leader) {  // the even CTA's full barriers track both CTAs' copies
+        for (uint32_t k = 0; k < (uint32_t)C::STAGES && k < it; ++k) {
+          const uint32_t j = it - 1 - k;
+          const unsigned long long t0 = gtimer();
+          while (!mbar_try(&full[j % C::STAGES], (j / C::STAGES) & 1)) {
+            if (gtimer() - t0 > WAIT_LIMIT_NS) { atomicOr(&g_watchdog, 2u); break; }
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      uint32_t it = 0;
+      int tc = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += npairs, ++tc) {
+        const int acc = tc & 1;
+        const uint32_t aph = (tc >> 1) & 1;
+        if (!mbar_wait(&tempty[acc], aph ^ 1, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        for (int kb = 0; kb < num_kb; ++kb, ++it) {
+          const int s = it % C::STAGES;
+          const uint32_t ph = (it / C::STAGES) & 1;
+          if (!mbar_wait(&full[s], ph, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t ad = sw128_desc(saddr(sA + s * C::A_BYTES));
+          const uint64_t bd = sw128_desc(saddr(sB + s * C::B_BYTES));
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            umma_pair(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), C::IDESC, (kb | k) != 0);
+          umma_commit_pair(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit_pair(&tfull[acc]);
+      }
+    }
+  } else {
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int row = (int)rank * BM + q * 32 + lane;
+    int tc = 0;
+    for (int tile = pair; tile < num_tiles; tile += npairs, ++tc) {
+      const int mb = tile % num_m, nb = tile / num_m;
+      const int acc = tc & 1;
+      const uint32_t aph = (tc >> 1) & 1;
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[acc], aph, abort_flag) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const int m = mb * 2 * BM + row;
+      for (int c = 0; c < BN; c += 32) {
+        const int n0 = nb * BN + c;
+        if (n0 >= N) break;
+        float v[32];
+        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN + c), v);
+        if (m < M) epi_chunk<bf16, 32>(e, m, n0, N, v);
+      }
+      tc_fence_before();
+      mbar_arrive_cluster(map_to(&tempty[acc], 0));
+    }
+  }
+  tc_fence_before();
+  __syncwarp();
+  cluster_sync_all();  // no CTA leaves while its peer may still address its TMEM or barriers
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(C::TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -292,6 +498,8 @@ bool init_driver() {
     if (g_sms <= 0) g_sms = 148;
     cudaFuncSetAttribute(k_gemm_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<128>::SMEM);
     cudaFuncSetAttribute(k_gemm_tc<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
+    cudaFuncSetAttribute(k_gemm_tc2<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<128>::SMEM);
+    cudaFuncSetAttribute(k_gemm_tc2<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<256>::SMEM);
   });
   return g_encode != nullptr;
 }
@@ -309,14 +517,15 @@ bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int ld, int 
   return r == CUDA_SUCCESS;
 }
 
-// Tile width choice: the fewest waves of 128 x BN tiles over the SMs,
-// ties to the wider tile (half the shared-memory traffic per FLOP).
-int pick_bn(int M, int N) {
+// Tile width choice: the fewest waves of rows_per_tile x BN tiles over the
+// available CTAs (or CTA pairs), ties to the wider tile (less shared-memory
+// traffic per FLOP).
+int pick_bn(int M, int N, int rows_per_tile, int slots) {
   double best = 1e30;
   int bn = 256;
   for (int cand : {256, 128}) {
-    const long long tiles = (long long)((M + BM - 1) / BM) * ((N + cand - 1) / cand);
-    const long long waves = (tiles + g_sms - 1) / g_sms;
+    const long long tiles = (long long)((M + rows_per_tile - 1) / rows_per_tile) * ((N + cand - 1) / cand);
+    const long long waves = (tiles + slots - 1) / slots;
     const double cost = (double)waves * cand;
     if (cost < best - 1e-9) { best = cost; bn = cand; }
   }
@@ -331,8 +540,20 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
   if (!init_driver()) return cudaErrorNotSupported;
   if (K % 8 != 0 || lda % 8 != 0 || ldw % 8 != 0 || N % 8 != 0) return cudaErrorInvalidValue;
   if (((uintptr_t)A & 15) || ((uintptr_t)W & 15)) return cudaErrorInvalidValue;
-  const int bn = pick_bn(M, N);
   CUtensorMap ma, mb;
+  if (M >= 2 * BM) {  // CTA pairs, 256-row tiles
+    const int pairs = g_sms / 2;
+    const int bn = pick_bn(M, N, 2 * BM, pairs);
+    if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, bn / 2)) return cudaErrorInvalidValue;
+    const long long tiles = (long long)((M + 2 * BM - 1) / (2 * BM)) * ((N + bn - 1) / bn);
+    const int grid = 2 * (int)(tiles < pairs ? tiles : pairs);
+    if (bn == 256)
+      k_gemm_tc2<256><<<grid, THREADS, Cfg2<256>::SMEM, s>>>(ma, mb, M, N, K, e);
+    else
+      k_gemm_tc2<128><<<grid, THREADS, Cfg2<128>::SMEM, s>>>(ma, mb, M, N, K, e);
+    return launched();
+  }
+  const int bn = pick_bn(M, N, BM, g_sms);
   if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, bn)) return cudaErrorInvalidValue;
   const long long tiles = (long long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
   const int grid = (int)(tiles < g_sms ? tiles : g_sms);

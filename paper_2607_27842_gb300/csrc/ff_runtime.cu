@@ -50,8 +50,11 @@ struct featfix_ctx {
   void *patches = nullptr, *pos = nullptr;
   float* mout = nullptr;
   float2* rope = nullptr;
-  // refresh history
+  // refresh history: per-block increments R_l and their sum over blocks
   void* ring = nullptr;
+  void* sring = nullptr;            // [S][E]: x_L - x_0 of each refresh step
+  void* x0buf = nullptr;            // block-0 input of the current step
+  void* shadow = nullptr;           // Verify arm: paid check on a copy
   int S = 0;
   // modulation: concatenated block weights and the per-trajectory tables
   void* wmod = nullptr;
@@ -636,6 +639,42 @@ Hist4 hist_ptrs(featfix_ctx* c, int l, int nt) {
   return h;
 }
 
+Hist4 sum_ptrs(featfix_ctx* c, int nt) {
+  Hist4 h = {{nullptr, nullptr, nullptr, nullptr}};
+  for (int j = 0; j < nt; ++j) h.p[j] = off(c->sring, (long long)(((c->head - j) % c->S + c->S) % c->S) * c->E, c->es);
+  return h;
+}
+
+// Paid check of a site in the Verify arm on a shadow copy of the step's
+// block-0 input: the per-block drafts chained up to each site, the exact
+// block from the same incoming state (Eq. 3), the logged discrepancy (Eq. 4),
+// then the draft continues (Verify forwards h_d).
+featfix_status verify_shadow(featfix_ctx* ctx, int i, int nt, const float* wf) {
+  const int L = ctx->L;
+  int last = -1;
+  for (int l = 0; l < L; ++l)
+    if (ctx->kinds[(size_t)i * L + l] == FEATFIX_PLAN_SITE) last = l;
+  if (last < 0) return FEATFIX_OK;
+  const size_t bytes = (size_t)ctx->E * ctx->es;
+  FF_CK(cudaMemcpyAsync(ctx->shadow, ctx->x0buf, bytes, cudaMemcpyDeviceToDevice, ctx->st));
+  for (int l = 0; l <= last; ++l) {
+    if (ctx->kinds[(size_t)i * L + l] == FEATFIX_PLAN_SITE) {
+      FF_TRY(exact_block(ctx, i, l, ctx->shadow, ctx->xa, nullptr));
+      ctx->cnt.paid_checks++;
+      const int slot = (int)ctx->log_sites.size();
+      if (slot >= ctx->max_logs) return fail(ctx, FEATFIX_ERR_STATE, "log overflow");
+      KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 3) * bytes);
+      FF_CK(launch_verify(ctx->dt, ctx->shadow, hist_ptrs(ctx, l, nt), wf, nt, ctx->xa, ctx->E, 1,
+                          ctx->dsums + 4 * slot, ctx->vws, ctx->st));
+      ctx->log_sites.push_back({i, l});
+    } else {
+      KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
+      FF_CK(launch_draft(ctx->dt, ctx->shadow, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
+    }
+  }
+  return FEATFIX_OK;
+}
+
 // One denoising step (modulations of step i ready): embedding, the L blocks
 // per the plan (exact / draft / paid site), final layer, sampler update.
 featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* cond) {
@@ -649,45 +688,64 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
   const bool refresh = ctx->isref[i] != 0;
   const bool vanilla = ctx->mode == FEATFIX_MODE_VANILLA;
   const size_t bytes = (size_t)ctx->E * ctx->es;
-  void* x = ctx->xa;
-  void* y = ctx->xb;
-  FF_TRY(embed(ctx, latent, cond, x));
+  FF_TRY(embed(ctx, latent, cond, ctx->x0buf));
   const int new_slot = (ctx->head + 1) % ctx->S;
   const int nt = ctx->keff[i] + 1;
   float wf[4];
   for (int j = 0; j < 4; ++j) wf[j] = (float)ctx->wts[(size_t)i * 4 + j];
-  for (int l = 0; l < L; ++l) {
-    for (auto& cp : ctx->caps)
-      if (cp.step == i && cp.layer == l && cp.in) FF_CK(cudaMemcpyAsync(cp.in, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
-    const unsigned char kind = ctx->kinds[(size_t)i * L + l];
-    if (kind == FEATFIX_PLAN_EXACT) {
-      void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, new_slot) : nullptr;
-      FF_TRY(exact_block(ctx, i, l, x, y, hist));
-      std::swap(x, y);
-    } else if (kind == FEATFIX_PLAN_DRAFT) {
-      KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
-      FF_CK(launch_draft(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
-    } else {
-      FF_TRY(exact_block(ctx, i, l, x, y, nullptr));
-      ctx->cnt.paid_checks++;
-      if (ctx->mode != FEATFIX_MODE_EXACT_ONLY) {
-        const int slot = (int)ctx->log_sites.size();
-        if (slot >= ctx->max_logs) return fail(ctx, FEATFIX_ERR_STATE, "log overflow");
-        const int wr = ctx->mode == FEATFIX_MODE_VERIFY ? 1 : 0;
-        KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 2 + wr) * bytes);
-        FF_CK(launch_verify(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, y, ctx->E, wr, ctx->dsums + 4 * slot, ctx->vws,
-                            ctx->st));
-        ctx->log_sites.push_back({i, l});
+  bool has_site = false, has_capture = false;
+  for (int l = 0; l < L; ++l) has_site |= ctx->kinds[(size_t)i * L + l] == FEATFIX_PLAN_SITE;
+  for (auto& cp : ctx->caps) has_capture |= cp.step == i;
+  const bool telescope = !refresh && !vanilla && !has_capture && !(ctx->flags & FEATFIX_FLAG_PER_BLOCK_DRAFT) &&
+                         (!has_site || ctx->mode == FEATFIX_MODE_VERIFY);
+  void* x = ctx->x0buf;
+  if (telescope) {
+    if (has_site) FF_TRY(verify_shadow(ctx, i, nt, wf));
+    KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
+    FF_CK(launch_draft(ctx->dt, x, sum_ptrs(ctx, nt), wf, nt, ctx->E, ctx->st));
+  } else {
+    // x0buf, then ping-pong xa / xb: x0buf stays the step's input for the
+    // refresh sum below
+    void* y = ctx->xa;
+    auto advance = [&]() {  // the block wrote y: it becomes the state
+      x = y;
+      y = (x == ctx->xa) ? ctx->xb : ctx->xa;
+    };
+    for (int l = 0; l < L; ++l) {
+      for (auto& cp : ctx->caps)
+        if (cp.step == i && cp.layer == l && cp.in) FF_CK(cudaMemcpyAsync(cp.in, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
+      const unsigned char kind = ctx->kinds[(size_t)i * L + l];
+      if (kind == FEATFIX_PLAN_EXACT) {
+        void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, new_slot) : nullptr;
+        FF_TRY(exact_block(ctx, i, l, x, y, hist));
+        advance();
+      } else if (kind == FEATFIX_PLAN_DRAFT) {
+        KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
+        FF_CK(launch_draft(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
+      } else {
+        FF_TRY(exact_block(ctx, i, l, x, y, nullptr));
+        ctx->cnt.paid_checks++;
+        if (ctx->mode != FEATFIX_MODE_EXACT_ONLY) {
+          const int slot = (int)ctx->log_sites.size();
+          if (slot >= ctx->max_logs) return fail(ctx, FEATFIX_ERR_STATE, "log overflow");
+          const int wr = ctx->mode == FEATFIX_MODE_VERIFY ? 1 : 0;
+          KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 2 + wr) * bytes);
+          FF_CK(launch_verify(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, y, ctx->E, wr, ctx->dsums + 4 * slot,
+                              ctx->vws, ctx->st));
+          ctx->log_sites.push_back({i, l});
+        }
+        if (ctx->mode != FEATFIX_MODE_VERIFY) {
+          advance();
+          ctx->cnt.forwarded++;
+        }
       }
-      if (ctx->mode != FEATFIX_MODE_VERIFY) {
-        std::swap(x, y);
-        ctx->cnt.forwarded++;
-      }
+      for (auto& cp : ctx->caps)
+        if (cp.step == i && cp.layer == l && cp.out) FF_CK(cudaMemcpyAsync(cp.out, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
     }
-    for (auto& cp : ctx->caps)
-      if (cp.step == i && cp.layer == l && cp.out) FF_CK(cudaMemcpyAsync(cp.out, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
   }
   if (refresh && !vanilla) {
+    KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+    FF_CK(launch_diff(ctx->dt, x, ctx->x0buf, off(ctx->sring, (long long)new_slot * ctx->E, ctx->es), ctx->E, ctx->st));
     ctx->head = new_slot;
     ctx->count = std::min(ctx->count + 1, ctx->S);
   }
@@ -741,7 +799,7 @@ featfix_status build_graph(featfix_ctx* ctx) {
 void free_all(featfix_ctx* c) {
   graph_reset(c);
   void* bufs[] = {c->xa, c->xb, c->xm, c->qkv, c->att, c->u1, c->big, c->patches, c->pos, c->mout, c->rope,
-                  c->ring, c->wmod, c->bmod, c->d_times, c->d_need, c->sin_tab, c->thid_tab, c->temb_tab,
+                  c->ring, c->sring, c->x0buf, c->shadow, c->wmod, c->bmod, c->d_times, c->d_need, c->sin_tab, c->thid_tab, c->temb_tab,
                   c->cs_all, c->cs_need, c->bmodtab, c->fmodtab, c->dsums, c->vws, c->g_lat, c->g_cond,
                   c->h_latent, c->h_cond};
   for (void* p : bufs)
@@ -841,6 +899,8 @@ featfix_status create_impl(featfix_ctx* ctx) {
   FF_CK(cudaStreamCreateWithFlags(&ctx->cap_st, cudaStreamNonBlocking));
   FF_TRY(alloc(ctx, &ctx->xa, T * C * es));
   FF_TRY(alloc(ctx, &ctx->xb, T * C * es));
+  FF_TRY(alloc(ctx, &ctx->x0buf, T * C * es));
+  FF_TRY(alloc(ctx, &ctx->shadow, T * C * es));
   FF_TRY(alloc(ctx, &ctx->xm, T * C * es));
   FF_TRY(alloc(ctx, &ctx->qkv, T * 3 * C * es));
   FF_TRY(alloc(ctx, &ctx->att, T * C * es));
@@ -872,8 +932,14 @@ featfix_status create_impl(featfix_ctx* ctx) {
 featfix_status schedule_buffers(featfix_ctx* ctx, int steps, int K, int mode, int n_sites) {
   const int es = ctx->es, C = ctx->C, Bm = ctx->Bm;
   const int S = K + 1;
-  if (ctx->ring && ctx->S != S) free_ptr(&ctx->ring);
-  if (!ctx->ring && mode != FEATFIX_MODE_VANILLA) FF_TRY(alloc(ctx, &ctx->ring, (size_t)ctx->L * S * ctx->E * es));
+  if (ctx->ring && ctx->S != S) {
+    free_ptr(&ctx->ring);
+    free_ptr(&ctx->sring);
+  }
+  if (!ctx->ring && mode != FEATFIX_MODE_VANILLA) {
+    FF_TRY(alloc(ctx, &ctx->ring, (size_t)ctx->L * S * ctx->E * es));
+    FF_TRY(alloc(ctx, &ctx->sring, (size_t)S * ctx->E * es));
+  }
   ctx->S = S;
   const int nlog = std::max(n_sites, 1);
   if (nlog > ctx->max_logs) {

@@ -21,6 +21,7 @@ DTYPE = {"f32": 0, "bf16": 1}
 SAMPLER = {"euler": 0, "ddim": 1}
 PLAN_EXACT, PLAN_DRAFT, PLAN_SITE = 0, 1, 2
 FLAG_TAYLOR_RECURSIVE = 1
+FLAG_PER_BLOCK_DRAFT = 2
 KCLASS = {"gemm": 0, "attention": 1, "draft": 2, "verify": 3, "other": 4}
 
 

@@ -133,16 +133,18 @@ def test_featfix_site_forwards_exact_output_bitwise(case):
     assert torch.equal(h, hf)
 
 
-def test_arms_bitwise(case):
+@pytest.mark.parametrize("flags", [0, ff.FLAG_PER_BLOCK_DRAFT], ids=["telescoped", "per_block"])
+def test_arms_bitwise(case, flags):
     """Exact-only == FeatFix; Verify == schedule without sites; all-refresh ==
-    vanilla; two runs identical."""
+    vanilla; two runs identical -- with drafted steps evaluated in one pass
+    and chained block by block."""
     wl = case.wl
     runs = {}
     for tag, mode, sites, refresh in (("featfix", "featfix", None, None), ("exact_only", "exact_only", None, None),
                                       ("verify", "verify", None, None), ("nosite", "featfix", (), None),
                                       ("allref", "featfix", (), tuple(range(wl.steps))),
                                       ("vanilla", "vanilla", None, None)):
-        case.schedule(mode, refresh=refresh, sites=sites)
+        case.schedule(mode, refresh=refresh, sites=sites, flags=flags)
         runs[tag] = case.sample(seed=5).clone()
         runs[tag + "_log"] = ff.featfix_get_log(case.ctx)
     assert torch.equal(runs["featfix"], runs["exact_only"])
@@ -155,10 +157,20 @@ def test_arms_bitwise(case):
     assert runs["vanilla_log"][1]["refresh_steps"] == wl.steps
     # same state at the first paid check in both arms -> same logged value
     assert runs["featfix_log"][0][0]["rel_l1"] == runs["verify_log"][0][0]["rel_l1"]
-    case.schedule("featfix")
+    case.schedule("featfix", flags=flags)
     again = case.sample(seed=5)
     assert torch.equal(again, runs["featfix"])
     assert ff.featfix_get_log(case.ctx)[0] == runs["featfix_log"][0]
+
+
+def test_telescoped_steps_match_per_block(case):
+    """A drafted step evaluated in one pass over the refresh sums
+    x_L - x_0 equals chaining the per-block drafts up to rounding."""
+    case.schedule("featfix")
+    a = case.sample(seed=7).cpu().numpy()
+    case.schedule("featfix", flags=ff.FLAG_PER_BLOCK_DRAFT)
+    b = case.sample(seed=7).cpu().numpy()
+    assert rel_l2(a, b) < (1e-5 if case.sh.dtype == "f32" else 1e-2)
 
 
 def test_call_order_errors(cuda):
