@@ -229,6 +229,23 @@ def run_reference(args, wl, rank):
 # our arm
 # ----------------------------------------------------------------------------
 
+def slowest_rank(dist, durations, device):
+    """Max over ranks of each timed duration: replicas run independently and
+    the job ends with its slowest rank (no data is exchanged)."""
+    if dist is None:
+        return list(durations)
+    import torch
+    t = torch.tensor(list(durations), dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
+def job_rate(units_per_rank, world, seconds):
+    """Whole-job throughput: the units every rank processed over the slowest
+    rank's time (weak scaling: per-rank work fixed)."""
+    return units_per_rank * world / seconds
+
+
 def profile_traffic():
     """DRAM bytes per launch of the dominant kernel from the committed ncu
     summary, when it was taken on the current kernel source (else None)."""
@@ -330,14 +347,9 @@ def main():
     barrier()
     e2e_s = time.perf_counter() - t0
 
-    ms_max, e2e_max = ms, e2e_s
-    if dist is not None:
-        t = torch.tensor([ms, e2e_s], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_max, e2e_max = float(t[0]), float(t[1])
-    steps_total = args.steps * wl.steps * world
-    value = steps_total / (ms_max / 1e3)
-    e2e = steps_total / e2e_max
+    ms_max, e2e_max = slowest_rank(dist, [ms, e2e_s], dev)
+    value = job_rate(args.steps * wl.steps, world, ms_max / 1e3)
+    e2e = job_rate(args.steps * wl.steps, world, e2e_max)
 
     hbm, tf_burst, tf_sus, src = peaks()
     g_ms, g_n, g_work = kt["gemm"]

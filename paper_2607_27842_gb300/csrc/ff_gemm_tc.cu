@@ -1,15 +1,15 @@
 // bf16 dense layers of the exact block (Eq. 1) on the 5th-generation tensor
 // cores: out = epilogue(A[M,K] W[N,K]^T).
 //
-// Persistent kernel, one CTA per SM, 6 warps:
+// Persistent kernel, one CTA per SM, 10 warps:
 //   warp 0      TMA producer: A and W tiles (128 and BN rows x 64 k, 128-byte
 //               swizzle) into a STAGES-deep shared-memory ring;
 //   warp 1      TMEM allocator and the single MMA-issuing thread:
 //               tcgen05.mma.cta_group::1.kind::f16 (M = 128, N = BN, K = 16),
 //               fp32 accumulators in TMEM, tcgen05.commit frees ring slots;
-//   warps 2..5  epilogue: tcgen05.ld of the accumulator (each warp its
-//               32-lane quarter), the fused bias / RoPE / GELU / gate /
-//               residual / history epilogue, 16-byte global stores.
+//   warps 2..9  epilogue: tcgen05.ld of the accumulator (each warp one
+//               32-lane quarter and one column half), the fused bias / RoPE /
+//               GELU / gate / residual / history epilogue, 16-byte stores.
 // Two TMEM accumulators (2 * BN columns) let the epilogue of tile i overlap
 // the main loop of tile i + 1.  Every mbarrier wait is bounded: on timeout
 // the CTA raises a watchdog flag, stops issuing work and releases its TMEM.
@@ -26,7 +26,7 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int THREADS = 192;
+constexpr int THREADS = 320;  // producer, MMA, 8 epilogue warps
 constexpr unsigned long long WAIT_LIMIT_NS = 4000000000ull;  // 4 s
 
 __device__ unsigned int g_watchdog;
@@ -195,7 +195,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 128);
+      mbar_init(&tempty[a], 256);
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -268,7 +268,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
     }
   } else {
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    // 8 epilogue warps: TMEM lane quarter q = warp % 4 (the quarter a warp
+    // may access), column half h of the tile
+    const int q = warp & 3;
+    const int h = (warp - 2) >> 2;
     const int row = q * 32 + lane;
     int tc = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++tc) {
@@ -281,7 +284,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       const int m = mb * BM + row;
-      for (int c = 0; c < BN; c += 32) {
+      for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
         const int n0 = nb * BN + c;
         if (n0 >= N) break;
         float v[32];
@@ -371,7 +374,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 2 * 128);
+      mbar_init(&tempty[a], 2 * 256);
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -445,6 +448,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     }
   } else {
     const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int h = (warp - 2) >> 2;  // column half of the tile
     const int row = (int)rank * BM + q * 32 + lane;
     int tc = 0;
     for (int tile = pair; tile < num_tiles; tile += npairs, ++tc) {
@@ -457,7 +461,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       const int m = mb * 2 * BM + row;
-      for (int c = 0; c < BN; c += 32) {
+      for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
         const int n0 = nb * BN + c;
         if (n0 >= N) break;
         float v[32];
@@ -541,7 +545,9 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
   if (K % 8 != 0 || lda % 8 != 0 || ldw % 8 != 0 || N % 8 != 0) return cudaErrorInvalidValue;
   if (((uintptr_t)A & 15) || ((uintptr_t)W & 15)) return cudaErrorInvalidValue;
   CUtensorMap ma, mb;
-  if (M >= 2 * BM) {  // CTA pairs, 256-row tiles
+  // Long reductions: CTA pairs (256-row tiles, each CTA stages half of W);
+  // measured faster than single CTAs only from K of about 8k on.
+  if (M >= 2 * BM && K >= 8192) {
     const int pairs = g_sms / 2;
     const int bn = pick_bn(M, N, 2 * BM, pairs);
     if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, bn / 2)) return cudaErrorInvalidValue;

@@ -157,12 +157,13 @@ def test_gemm_plain_and_bias(cuda, dtype, M, N, K):
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
-def test_gemm_fused_epilogues(cuda, dtype):
-    M, N, K, rpb = 384, 256, 192, 128
+@pytest.mark.parametrize("M,N,K,rpb", [(384, 256, 192, 128),      # row-wise epilogue
+                                       (1100, 520, 192, 500)])    # narrow output: transposed tiles, ragged
+def test_gemm_fused_epilogues(cuda, dtype, M, N, K, rpb):
     a = randn((M, K), dtype, 4)
     w = randn((N, K), dtype, 5, 0.08)
     bias = randn(N, dtype, 6, 0.3)
-    gate = randn((3, 2 * N), "f32", 7)
+    gate = randn(((M + rpb - 1) // rpb, 2 * N), "f32", 7)
     resid = randn((M, N), dtype, 8)
     out = torch.empty((M, N), dtype=TD[dtype], device=cuda)
     hout = torch.empty_like(out)
