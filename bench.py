@@ -251,7 +251,7 @@ def profile_traffic():
     summary, when it was taken on the current kernel source (else None)."""
     path = os.path.join(ROOT, "profiles", "gemm_tc_dit_xl2.md")
     src = b""
-    for f in ("ff_gemm_tc.cu", "ff_common.cuh"):
+    for f in ("ff_gemm_tc.cu", "ff_tc.cuh", "ff_common.cuh"):
         with open(os.path.join(ROOT, "paper_2607_27842_gb300", "csrc", f), "rb") as fh:
             src += fh.read()
     digest = hashlib.sha256(src).hexdigest()[:16]

@@ -22,7 +22,7 @@ LIB = os.path.join(HERE, "libfeatfix.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include"), "-I", CSRC]
-SOURCES = ["ff_elementwise.cu", "ff_simt.cu", "ff_gemm_tc.cu", "ff_attention.cu", "ff_runtime.cu", "ff_ops.cu", "ff_noalloc.cu"]
+SOURCES = ["ff_elementwise.cu", "ff_simt.cu", "ff_gemm_tc.cu", "ff_attention.cu", "ff_attention_tc.cu", "ff_runtime.cu", "ff_ops.cu", "ff_noalloc.cu"]
 
 
 def nvcc():

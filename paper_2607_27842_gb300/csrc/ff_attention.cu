@@ -1,5 +1,7 @@
 // Non-causal multi-head attention inside the exact block (Eq. 1) over the
-// joint [text ; image] token sequence of each sample.
+// joint [text ; image] token sequence of each sample.  bf16 runs on the
+// tcgen05 kernel of ff_attention_tc.cu when the fused qkv layout allows;
+// otherwise (and for head widths 32):
 //
 // bf16: flash-style kernel on warp-level mma.sync (m16n8k16, fp32
 // accumulate): 64 queries per CTA (16 per warp), keys/values streamed in
@@ -255,8 +257,15 @@ cudaError_t attn_mma_t(const AttnArgs& a, cudaStream_t s) {
 }  // namespace
 
 cudaError_t attention(DType dt, const AttnArgs& a, cudaStream_t s) {
-  if (a.B <= 0 || a.Nt + a.Ni <= 0) return cudaSuccess;
+  if (a.B <= 0 || a.H <= 0 || a.Nt + a.Ni <= 0) return cudaSuccess;
   if (dt == BF16) {
+    // tensor cores (tcgen05) when the layout allows and the sequence is long
+    // enough to amortise the per-CTA set-up (measured: slower than the
+    // mma.sync kernel at 256 tokens, faster from a few thousand on)
+    if (a.Nt + a.Ni >= 1024) {
+      const cudaError_t e = attention_tc(a, s);
+      if (e != cudaErrorInvalidValue && e != cudaErrorNotSupported) return e;
+    }
     switch (a.hd) {
       case 32: return attn_mma_t<32>(a, s);
       case 64: return attn_mma_t<64>(a, s);

@@ -263,6 +263,8 @@ struct AttnArgs {
   int B, Nt, Ni, H, hd;
 };
 cudaError_t attention(DType dt, const AttnArgs& a, cudaStream_t s);
+cudaError_t attention_tc(const AttnArgs& a, cudaStream_t s);
+unsigned int attention_tc_watchdog_take();
 cudaError_t attention_simt(DType dt, const AttnArgs& a, cudaStream_t s);
 
 }  // namespace ff

@@ -14,6 +14,7 @@
 // the main loop of tile i + 1.  Every mbarrier wait is bounded: on timeout
 // the CTA raises a watchdog flag, stops issuing work and releases its TMEM.
 #include "ff_common.cuh"
+#include "ff_tc.cuh"
 
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -27,9 +28,13 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr int THREADS = 320;  // producer, MMA, 8 epilogue warps
-constexpr unsigned long long WAIT_LIMIT_NS = 4000000000ull;  // 4 s
+using namespace tc;
 
 __device__ unsigned int g_watchdog;
+
+__device__ __forceinline__ bool mbar_wait_g(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
+  return mbar_wait(b, parity, abort_flag, &g_watchdog);
+}
 
 template <int BN> struct Cfg {
   static constexpr int STAGES = BN >= 256 ? 4 : 6;
@@ -43,129 +48,6 @@ template <int BN> struct Cfg {
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                                     ((uint32_t)(BM >> 4) << 24);
 };
-
-__device__ __forceinline__ uint32_t saddr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ unsigned long long gtimer() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(saddr(b)), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* b, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(saddr(b)), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(saddr(b)) : "memory");
-}
-// try_wait with a suspend-time hint: the waiting thread sleeps in hardware
-// (up to ~0.1 ms) instead of re-issuing the poll.
-__device__ __forceinline__ bool mbar_try(uint64_t* b, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}\n"
-      : "=r"(ok)
-      : "r"(saddr(b)), "r"(parity), "r"(100000u)
-      : "memory");
-  return ok != 0;
-}
-// Bounded wait on phase `parity`; false (and the CTA abort flag raised) on
-// timeout or when another role already aborted.
-__device__ __noinline__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
-  if (mbar_try(b, parity)) return true;
-  const unsigned long long t0 = gtimer();
-  for (uint32_t it = 1;; ++it) {
-    if (mbar_try(b, parity)) return true;
-    if ((it & 63) == 0) {
-      if (*abort_flag) return false;
-      if (gtimer() - t0 > WAIT_LIMIT_NS) {
-        *abort_flag = 1;
-        atomicOr(&g_watchdog, 1u);
-        return false;
-      }
-    }
-  }
-}
-
-__device__ __forceinline__ void tma_load(const CUtensorMap* tm, uint64_t* bar, void* dst, int x, int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
-          saddr(dst)),
-      "l"((uint64_t)tm), "r"(x), "r"(y), "r"(saddr(bar))
-      : "memory");
-}
-
-// ---- CTA-pair (2-SM) helpers --------------------------------------------------
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-// shared::cluster address of the same object in CTA `rank` of the cluster
-__device__ __forceinline__ uint32_t map_to(const void* p, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr(p)), "r"(rank));
-  return r;
-}
-__device__ __forceinline__ void cluster_sync_all() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-// TMA load into this CTA's shared memory that completes on an mbarrier of
-// either CTA of the pair (shared::cluster address).
-__device__ __forceinline__ void tma_load_pair(const CUtensorMap* tm, uint32_t bar_cluster, void* dst, int x, int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
-      "[%4];" ::"r"(saddr(dst)),
-      "l"((uint64_t)tm), "r"(x), "r"(y), "r"(bar_cluster)
-      : "memory");
-}
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
-}
-
-// Shared-memory matrix descriptor, K-major operand with 128-byte swizzle:
-// start address >> 4 (bits 0-13), leading offset 1 (unused for swizzled
-// K-major), stride offset 1024 B between 8-row groups (bits 32-45),
-// descriptor version 1 (bits 46-47), swizzle mode 2 = 128B (bits 61-63).
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
-  uint64_t d = (uint64_t)((addr & 0x3FFFF) >> 4);
-  d |= (uint64_t)1 << 16;
-  d |= (uint64_t)(1024 >> 4) << 32;
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;
-  return d;
-}
-
-__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
-          d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(accum));
-}
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(saddr(bar))
-               : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
-      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
-        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
-        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
 
 template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
@@ -222,7 +104,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_g(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
           mbar_expect_tx(&full[s], C::STAGE_BYTES);
           tma_load(&tmA, &full[s], sA + s * C::A_BYTES, kb * BK, mb * BM);
           tma_load(&tmB, &full[s], sB + s * C::B_BYTES, kb * BK, nb * BN);
@@ -246,13 +128,13 @@ __global__ void __launch_bounds__(THREADS, 1)
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++tc) {
         const int acc = tc & 1;
         const uint32_t aph = (tc >> 1) & 1;
-        if (!mbar_wait(&tempty[acc], aph ^ 1, abort_flag)) break;
+        if (!mbar_wait_g(&tempty[acc], aph ^ 1, abort_flag)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait(&full[s], ph, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_g(&full[s], ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
           const uint64_t ad = sw128_desc(saddr(sA + s * C::A_BYTES));
           const uint64_t bd = sw128_desc(saddr(sB + s * C::B_BYTES));
@@ -279,7 +161,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int acc = tc & 1;
       const uint32_t aph = (tc >> 1) & 1;
       int ok = 1;
-      if (lane == 0) ok = mbar_wait(&tfull[acc], aph, abort_flag) ? 1 : 0;
+      if (lane == 0) ok = mbar_wait_g(&tfull[acc], aph, abort_flag) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
@@ -402,7 +284,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_g(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
           if (leader) mbar_expect_tx(&full[s], 2 * C::STAGE_BYTES);
           const uint32_t fb = map_to(&full[s], 0);
           tma_load_pair(&tmA, fb, sA + s * C::A_BYTES, kb * BK, mb * 2 * BM + (int)rank * BM);
@@ -427,13 +309,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       for (int tile = pair; tile < num_tiles && ok; tile += npairs, ++tc) {
         const int acc = tc & 1;
         const uint32_t aph = (tc >> 1) & 1;
-        if (!mbar_wait(&tempty[acc], aph ^ 1, abort_flag)) break;
+        if (!mbar_wait_g(&tempty[acc], aph ^ 1, abort_flag)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait(&full[s], ph, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_g(&full[s], ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
           const uint64_t ad = sw128_desc(saddr(sA + s * C::A_BYTES));
           const uint64_t bd = sw128_desc(saddr(sB + s * C::B_BYTES));
@@ -456,7 +338,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       const int acc = tc & 1;
       const uint32_t aph = (tc >> 1) & 1;
       int ok = 1;
-      if (lane == 0) ok = mbar_wait(&tfull[acc], aph, abort_flag) ? 1 : 0;
+      if (lane == 0) ok = mbar_wait_g(&tfull[acc], aph, abort_flag) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();

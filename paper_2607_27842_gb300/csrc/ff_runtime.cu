@@ -1182,8 +1182,8 @@ featfix_status featfix_sample_host(featfix_ctx* ctx, unsigned long long seed, in
 featfix_status featfix_get_log(featfix_ctx* ctx, featfix_site_log* out, int cap, int* n, featfix_counters* counters) {
   if (!ctx) return FEATFIX_ERR_INVALID_ARG;
   FF_CK(cudaStreamSynchronize(ctx->user_st));
-  const unsigned int wd = gemm_tc_watchdog_take();
-  if (wd) return fail(ctx, FEATFIX_ERR_CUDA, "tensor-core GEMM watchdog fired (code " + std::to_string(wd) + ")");
+  const unsigned int wd = gemm_tc_watchdog_take() | (attention_tc_watchdog_take() << 8);
+  if (wd) return fail(ctx, FEATFIX_ERR_CUDA, "tensor-core kernel watchdog fired (code " + std::to_string(wd) + ")");
   const int avail = (int)ctx->log_sites.size();
   if (n) *n = avail;
   if (counters) *counters = ctx->cnt;
