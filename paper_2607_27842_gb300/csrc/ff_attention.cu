@@ -259,13 +259,9 @@ cudaError_t attn_mma_t(const AttnArgs& a, cudaStream_t s) {
 cudaError_t attention(DType dt, const AttnArgs& a, cudaStream_t s) {
   if (a.B <= 0 || a.H <= 0 || a.Nt + a.Ni <= 0) return cudaSuccess;
   if (dt == BF16) {
-    // tensor cores (tcgen05) when the layout allows and the sequence is long
-    // enough to amortise the per-CTA set-up (measured: slower than the
-    // mma.sync kernel at 256 tokens, faster from a few thousand on)
-    if (a.Nt + a.Ni >= 1024) {
-      const cudaError_t e = attention_tc(a, s);
-      if (e != cudaErrorInvalidValue && e != cudaErrorNotSupported) return e;
-    }
+    // tensor cores (tcgen05) whenever the layout allows
+    const cudaError_t e = attention_tc(a, s);
+    if (e != cudaErrorInvalidValue && e != cudaErrorNotSupported) return e;
     switch (a.hd) {
       case 32: return attn_mma_t<32>(a, s);
       case 64: return attn_mma_t<64>(a, s);

@@ -1,20 +1,23 @@
 // Non-causal attention softmax(q k^T / sqrt(d)) v of the exact block (Eq. 1)
 // on the 5th-generation tensor cores, bf16 in, fp32 accumulate.
 //
-// One CTA per (sample, head, 128-query tile), 6 warps:
-//   warp 0     TMA producer: the query tile once, key / value tiles of 128
-//              tokens into a 2-stage ring, straight from the fused qkv
+// One CTA per (sample, head, pair of 128-query tiles), 10 warps:
+//   warp 0     TMA producer: both query tiles once, then key and value tiles
+//              of 128 tokens into separate rings, straight from the fused qkv
 //              activation (3-D tensor map: head width, head slot, row; the
 //              head width is zero-padded to a multiple of 64 by the map);
-//   warp 1     TMEM allocator and MMA issuer: S = Q K^T into one of two TMEM
-//              score buffers (tcgen05.mma, both operands K-major), then
-//              O += P V into the TMEM output accumulator (P K-major from
-//              shared memory, V MN-major straight from its tile);
-//   warps 2-5  softmax: each thread owns one query row (its TMEM lane):
-//              row max, exp2, row sum, P written as bf16 into shared memory
-//              in the 128-byte-swizzled operand layout; the output row is
-//              rescaled in TMEM only when the running max grew by more than
-//              2^8 (the normalisation divides by the same stale max).
+//   warp 1     TMEM allocator and MMA issuer.  Per key tile j and query tile
+//              i: S_i = Q_i K_j^T into TMEM (both operands K-major from shared
+//              memory), then O_i += P_i V_j with P_i read from TMEM (where the
+//              softmax wrote it over S_i) and V MN-major from its TMA tile.
+//              S_i for tile j + 1 is issued right behind O_i's update for
+//              tile j, so one query tile's softmax overlaps the other's MMAs;
+//   warps 2-5  softmax of query tile 0, warps 6-9 of query tile 1: each
+//              thread owns one query row (its TMEM lane): row max, exp2, row
+//              sum, P as bf16 pairs back into TMEM; O is rescaled in TMEM only
+//              when the running max grew by more than 2^8 (the final division
+//              uses the same stale max, so the result is unchanged).
+// TMEM columns: S_0 [0,128), S_1 [128,256), O_0 [256,384), O_1 [384,512).
 // Keys of a sample lie in up to two row segments (text rows, image rows of
 // the stream-major token layout); tiles never straddle a segment and keys
 // past a segment's end are masked.
@@ -33,11 +36,11 @@ namespace {
 
 using namespace tc;
 
-constexpr int AQ = 128;        // queries per CTA (MMA M)
+constexpr int AQ = 128;        // queries per tile (MMA M)
 constexpr int AKV = 128;       // keys per tile (MMA N of S, K of P V)
-constexpr int ATHREADS = 192;
-constexpr int KV_STAGES = 2;
+constexpr int ATHREADS = 320;
 constexpr float RESCALE_LOG2 = 8.0f;
+constexpr size_t SMEM_LIMIT = 232448;  // opt-in dynamic shared memory per block
 
 __device__ unsigned int g_attn_watchdog;
 
@@ -49,16 +52,20 @@ template <int D> struct ACfg {
   static constexpr int NBOX = D <= 64 ? 1 : 2;           // 64-wide column boxes per tile row
   static constexpr int DK = (D + 15) / 16 * 16;          // q k^T reduction width and P V output width
   static constexpr uint32_t BOX = 128 * 128;             // one [128 rows x 64] bf16 box, 16 KB
-  static constexpr uint32_t Q_BYTES = NBOX * BOX;
-  static constexpr uint32_t P_BYTES = 2 * BOX;           // [128 queries x 128 keys] bf16
-  static constexpr uint32_t KV_BYTES = 2 * NBOX * BOX;   // K tile + V tile
-  static constexpr size_t SMEM = 1024 + Q_BYTES + P_BYTES + (size_t)KV_STAGES * KV_BYTES + 256;
-  static constexpr uint32_t TMEM_O = 2 * AKV;            // columns [0,256) scores x2, then O
-  // kind::f16, D fp32, A/B bf16; S: both K-major, N = 128; O: B (V) MN-major (bit 16), N = DK
+  static constexpr uint32_t TILE = NBOX * BOX;           // one Q, K or V tile
+  static constexpr int NST = (int)((SMEM_LIMIT - 1024 - 512 - 2 * (size_t)TILE) / TILE);
+  static constexpr int KST = NST >= 8 ? 4 : (NST + 1) / 2;  // key ring depth
+  static constexpr int VST = NST >= 8 ? 4 : NST / 2;        // value ring depth
+  static constexpr size_t SMEM = 1024 + (size_t)(2 + KST + VST) * TILE + 512;
+  static constexpr uint32_t TMEM_O = 2 * AKV;
+  // kind::f16, D fp32, A/B bf16; S: both K-major, N = 128; O: A (P) from
+  // TMEM, B (V) MN-major (bit 16), N = DK
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(AKV >> 3) << 17) |
                                       ((uint32_t)(AQ >> 4) << 24);
   static constexpr uint32_t IDESC_O = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((uint32_t)(DK >> 3) << 17) |
                                       ((uint32_t)(AQ >> 4) << 24);
+  static_assert(KST >= 2 && VST >= 1, "shared memory too small for the key/value rings");
+  static_assert(SMEM <= SMEM_LIMIT, "shared memory budget");
 };
 
 // MN-major operand with 128-byte swizzle: 64 contiguous elements (128 B) per
@@ -74,6 +81,49 @@ __device__ __forceinline__ uint64_t sw128_desc_mn(uint32_t addr, uint32_t lbo) {
   return d;
 }
 
+// D[tmem] (+)= A[tmem] * B[smem]: A is read from TMEM (row m = lane m, two
+// bf16 per 32-bit column along K)
+__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(
+          d_tmem),
+      "r"(a_tmem), "l"(b), "r"(idesc), "r"(accum));
+}
+
+// 64 consecutive 32-bit TMEM columns of this warp's 32 lanes, waited for in
+// the same statement so no use of the registers can precede the wait
+__device__ __forceinline__ void tmem_ld64w(uint32_t taddr, uint32_t (&r)[64]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];\n"
+      "tcgen05.wait::ld.sync.aligned;\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+        "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]),
+        "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]),
+        "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};\n" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]),
+        "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]),
+        "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ void tma_load3(const CUtensorMap* tm, uint64_t* bar, void* dst, int x, int y, int z) {
   asm volatile(
       "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
@@ -84,7 +134,7 @@ __device__ __forceinline__ void tma_load3(const CUtensorMap* tm, uint64_t* bar, 
 
 // Row segments of sample b: text rows [b*Nt, b*Nt + Nt), image rows
 // [B*Nt + b*Ni, ... + Ni).  Tile t of the sample's sequence: first row and
-// number of valid rows.
+// number of valid rows (<= 0 for a tile past the sequence end).
 struct SegTile {
   int row0, valid;
 };
@@ -101,35 +151,40 @@ __global__ void __launch_bounds__(ATHREADS, 1)
   using C = ACfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQ = smem;
-  uint8_t* sP = sQ + C::Q_BYTES;
-  uint8_t* sKV = sP + C::P_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + KV_STAGES * C::KV_BYTES);
+  uint8_t* sQ = smem;                        // 2 tiles
+  uint8_t* sK = sQ + 2 * C::TILE;            // KST tiles
+  uint8_t* sV = sK + C::KST * C::TILE;       // VST tiles
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + C::VST * C::TILE);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;
-  uint64_t* kv_empty = kv_full + KV_STAGES;
-  uint64_t* s_full = kv_empty + KV_STAGES;
-  uint64_t* p_ready = s_full + 2;
-  uint64_t* o_done = p_ready + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_done + 1);
+  uint64_t* k_full = q_full + 1;
+  uint64_t* k_empty = k_full + C::KST;
+  uint64_t* v_full = k_empty + C::KST;
+  uint64_t* v_empty = v_full + C::VST;
+  uint64_t* s_full = v_empty + C::VST;       // per query tile
+  uint64_t* p_ready = s_full + 2;            // per query tile
+  uint64_t* o_final = p_ready + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_final + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int h = blockIdx.y, b = blockIdx.z;
   const int nkv = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;
-  const SegTile qs = seg_tile(a, b, qt);
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < KV_STAGES; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+    for (int s = 0; s < C::KST; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < C::VST; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
       mbar_init(&p_ready[i], 128);
     }
-    mbar_init(o_done, 1);
+    mbar_init(o_final, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQKV) : "memory");
@@ -146,150 +201,193 @@ __global__ void __launch_bounds__(ATHREADS, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      // query tile: head slot h
-      mbar_expect_tx(q_full, C::Q_BYTES);
-      for (int bx = 0; bx < C::NBOX; ++bx) tma_load3(&tmQKV, q_full, sQ + bx * C::BOX, 64 * bx, h, qs.row0);
+      mbar_expect_tx(q_full, 2 * C::TILE);
+      for (int i = 0; i < 2; ++i) {
+        const SegTile qs = seg_tile(a, b, 2 * blockIdx.x + i);
+        for (int bx = 0; bx < C::NBOX; ++bx) tma_load3(&tmQKV, q_full, sQ + i * C::TILE + bx * C::BOX, 64 * bx, h, qs.row0);
+      }
+      int nk = 0, nv = 0;
       for (int j = 0; j < nkv; ++j) {
-        const int s = j % KV_STAGES;
-        const uint32_t ph = (j / KV_STAGES) & 1;
-        if (!wait_a(&kv_empty[s], ph ^ 1, abort_flag)) break;
         const SegTile ks = seg_tile(a, b, j);
-        uint8_t* kdst = sKV + s * C::KV_BYTES;
-        uint8_t* vdst = kdst + C::NBOX * C::BOX;
-        mbar_expect_tx(&kv_full[s], C::KV_BYTES);
-        for (int bx = 0; bx < C::NBOX; ++bx) {
-          tma_load3(&tmQKV, &kv_full[s], kdst + bx * C::BOX, 64 * bx, a.H + h, ks.row0);
-          tma_load3(&tmQKV, &kv_full[s], vdst + bx * C::BOX, 64 * bx, 2 * a.H + h, ks.row0);
-        }
+        const int sk = j % C::KST, sv = j % C::VST;
+        if (!wait_a(&k_empty[sk], ((j / C::KST) & 1) ^ 1, abort_flag)) break;
+        mbar_expect_tx(&k_full[sk], C::TILE);
+        for (int bx = 0; bx < C::NBOX; ++bx)
+          tma_load3(&tmQKV, &k_full[sk], sK + sk * C::TILE + bx * C::BOX, 64 * bx, a.H + h, ks.row0);
+        ++nk;
+        if (!wait_a(&v_empty[sv], ((j / C::VST) & 1) ^ 1, abort_flag)) break;
+        mbar_expect_tx(&v_full[sv], C::TILE);
+        for (int bx = 0; bx < C::NBOX; ++bx)
+          tma_load3(&tmQKV, &v_full[sv], sV + sv * C::TILE + bx * C::BOX, 64 * bx, 2 * a.H + h, ks.row0);
+        ++nv;
+      }
+      // Copies still in flight complete on their full barriers; wait for the
+      // last ring's worth of each so none lands after the CTA exits.
+      for (int k = 0; k < C::KST && k < nk; ++k) {
+        const int j = nk - 1 - k;
+        const unsigned long long t0 = gtimer();
+        while (!mbar_try(&k_full[j % C::KST], (j / C::KST) & 1))
+          if (gtimer() - t0 > WAIT_LIMIT_NS) { atomicOr(&g_attn_watchdog, 2u); break; }
+      }
+      for (int k = 0; k < C::VST && k < nv; ++k) {
+        const int j = nv - 1 - k;
+        const unsigned long long t0 = gtimer();
+        while (!mbar_try(&v_full[j % C::VST], (j / C::VST) & 1))
+          if (gtimer() - t0 > WAIT_LIMIT_NS) { atomicOr(&g_attn_watchdog, 2u); break; }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       bool ok = wait_a(q_full, 0, abort_flag);
-      const uint64_t qd = sw128_desc(saddr(sQ));
-      const uint64_t pd = sw128_desc(saddr(sP));
-      for (int j = 0; j <= nkv && ok; ++j) {
-        if (j < nkv) {  // S_j = Q K_j^T into score buffer j % 2
-          const int s = j % KV_STAGES;
-          if (!wait_a(&kv_full[s], (j / KV_STAGES) & 1, abort_flag)) break;
-          tc_fence_after();
-          const uint64_t kd = sw128_desc(saddr(sKV + s * C::KV_BYTES));
+      const uint64_t qd0 = sw128_desc(saddr(sQ)), qd1 = sw128_desc(saddr(sQ + C::TILE));
+      // S_i = Q_i K_j^T (DK / 16 steps of 16 along the head width: box k / 4,
+      // +32 B per step inside the box), then arrive on s_full[i]
+      auto issue_s = [&](int i, int j) {
+        const uint64_t kd = sw128_desc(saddr(sK + (j % C::KST) * C::TILE));
+        const uint64_t qd = i ? qd1 : qd0;
 #pragma unroll
-          for (int k = 0; k < C::DK / 16; ++k) {
-            // 16-wide k step k: box k / 4, +32 B per step inside the box
-            const uint64_t off = (uint64_t)((k >> 2) * (C::BOX >> 4) + 2 * (k & 3));
-            umma(tmem + (uint32_t)((j & 1) * AKV), qd + off, kd + off, C::IDESC_S, k != 0);
-          }
-          umma_commit(&s_full[j & 1]);
+        for (int k = 0; k < C::DK / 16; ++k) {
+          const uint64_t off = (uint64_t)((k >> 2) * (C::BOX >> 4) + 2 * (k & 3));
+          umma(tmem + (uint32_t)(i * AKV), qd + off, kd + off, C::IDESC_S, k != 0);
         }
-        if (j >= 1) {  // O += P_{j-1} V_{j-1}
-          const int jp = j - 1, s = jp % KV_STAGES;
-          if (!wait_a(&p_ready[jp & 1], (jp >> 1) & 1, abort_flag)) break;
+        umma_commit(&s_full[i]);
+      };
+      if (ok) ok = wait_a(&k_full[0], 0, abort_flag);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        issue_s(1, 0);
+        umma_commit(&k_empty[0]);
+      }
+      for (int j = 0; j < nkv && ok; ++j) {
+        const int sv = j % C::VST;
+        if (!wait_a(&v_full[sv], (j / C::VST) & 1, abort_flag)) break;
+        const uint32_t vaddr = saddr(sV + sv * C::TILE);
+        for (int i = 0; i < 2 && ok; ++i) {
+          if (!wait_a(&p_ready[i], j & 1, abort_flag)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t vaddr = saddr(sKV + s * C::KV_BYTES + C::NBOX * C::BOX);
+          // O_i += P_i V_j: 16 keys per step = 8 TMEM columns of P, 2 groups
+          // of 8 value rows (2 KB) of the MN-major V tile
 #pragma unroll
           for (int k = 0; k < AKV / 16; ++k) {
-            // P: K-major, keys 64 per box; V: MN-major, 16 keys = 2 groups of 8 rows (2 KB)
-            const uint64_t poff = (uint64_t)((k >> 2) * (C::BOX >> 4) + 2 * (k & 3));
             const uint64_t vd = sw128_desc_mn(vaddr + (uint32_t)k * 2048u, C::BOX);
-            umma(tmem + C::TMEM_O, pd + poff, vd, C::IDESC_O, (jp | k) != 0);
+            umma_ts(tmem + C::TMEM_O + (uint32_t)(i * AKV), tmem + (uint32_t)(i * AKV + k * 8), vd, C::IDESC_O,
+                    (j | k) != 0);
           }
-          umma_commit(o_done);
-          umma_commit(&kv_empty[s]);
+          if (j + 1 < nkv) {
+            if (i == 0) {
+              if (!wait_a(&k_full[(j + 1) % C::KST], ((j + 1) / C::KST) & 1, abort_flag)) { ok = false; break; }
+              tc_fence_after();
+            }
+            issue_s(i, j + 1);  // behind O_i's update: the MMA pipe reads P_i before S_i is overwritten
+            if (i == 1) umma_commit(&k_empty[(j + 1) % C::KST]);
+          }
         }
+        if (!ok) break;
+        umma_commit(&v_empty[sv]);
       }
+      if (ok) umma_commit(o_final);
     }
   } else {
-    // softmax: row r of the tile = TMEM lane r
+    // softmax of query tile i: row r of the tile = TMEM lane r
+    const int i = (warp - 2) >> 2;
     const int q = warp & 3;
     const int r = q * 32 + lane;
-    const uint32_t lane_base = tmem + ((uint32_t)(q * 32) << 16);
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const uint32_t s_col = tmem + lane_off + (uint32_t)(i * AKV);
+    const uint32_t o_col = tmem + lane_off + C::TMEM_O + (uint32_t)(i * AKV);
+    const SegTile qs = seg_tile(a, b, 2 * blockIdx.x + i);
     float m = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int j = 0; j < nkv && ok; ++j) {
-      const SegTile ks = seg_tile(a, b, j);
+    for (int j = 0; j < nkv; ++j) {
+      const int valid = seg_tile(a, b, j).valid;
       int w = 1;
-      if (lane == 0) w = wait_a(&s_full[j & 1], (j >> 1) & 1, abort_flag) ? 1 : 0;
+      if (lane == 0) w = wait_a(&s_full[i], j & 1, abort_flag) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
       tc_fence_after();
-      const uint32_t sbase = lane_base + (uint32_t)((j & 1) * AKV);
-      float mx = -INFINITY;
+      float v[AKV];
+      {
+        uint32_t t[64];
+        tmem_ld64w(s_col, t);
 #pragma unroll
-      for (int c = 0; c < AKV / 32; ++c) {
-        float v[32];
-        tmem_ld32(sbase + (uint32_t)(c * 32), v);
+        for (int e = 0; e < 64; ++e) v[e] = __uint_as_float(t[e]);
+        tmem_ld64w(s_col + 64, t);
 #pragma unroll
-        for (int e = 0; e < 32; ++e)
-          if (c * 32 + e < ks.valid) mx = fmaxf(mx, v[e] * scale_log2);
+        for (int e = 0; e < 64; ++e) v[64 + e] = __uint_as_float(t[e]);
       }
-      const float m_new = fmaxf(m, mx);
+      if (valid < AKV) {
+#pragma unroll
+        for (int e = 0; e < AKV; ++e)
+          if (e >= valid) v[e] = -INFINITY;
+      }
+      // row max as a tree (depth 7)
+      float mx[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e)
+        mx[e] = fmaxf(fmaxf(fmaxf(v[e], v[e + 16]), fmaxf(v[e + 32], v[e + 48])),
+                      fmaxf(fmaxf(v[e + 64], v[e + 80]), fmaxf(v[e + 96], v[e + 112])));
+#pragma unroll
+      for (int s = 8; s >= 1; s >>= 1)
+#pragma unroll
+        for (int e = 0; e < s; ++e) mx[e] = fmaxf(mx[e], mx[e + s]);
+      const float m_new = fmaxf(m, mx[0] * scale_log2);
       const bool grow = m_new > m + RESCALE_LOG2;  // also true on the first tile
       const float m_use = grow ? m_new : m;
-      const float alpha = grow ? exp2f(m - m_new) : 1.0f;
-      if (j >= 1) {  // O and the P buffer are free once P_{j-1} V_{j-1} completed
-        int w2 = 1;
-        if (lane == 0) w2 = wait_a(o_done, (j - 1) & 1, abort_flag) ? 1 : 0;
-        if (!__shfl_sync(0xffffffffu, w2, 0)) { ok = false; break; }
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, grow)) {
-#pragma unroll
-          for (int c = 0; c < C::DK / 16; ++c) {
-            float o[16];
-            tmem_ld16(lane_base + C::TMEM_O + (uint32_t)(c * 16), o);
-#pragma unroll
-            for (int e = 0; e < 16; ++e) o[e] *= alpha;
-            tmem_st16(lane_base + C::TMEM_O + (uint32_t)(c * 16), o);
-          }
-        }
-      }
-      l *= alpha;
-      m = m_use;
-      // P row: 128 keys as bf16, 16-byte chunks swizzled by row (128B swizzle)
-#pragma unroll
-      for (int c = 0; c < AKV / 32; ++c) {
-        float v[32];
-        tmem_ld32(sbase + (uint32_t)(c * 32), v);
-        uint32_t pk[16];
-#pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          const float p0 = (c * 32 + e < ks.valid) ? exp2f(v[e] * scale_log2 - m) : 0.f;
-          const float p1 = (c * 32 + e + 1 < ks.valid) ? exp2f(v[e + 1] * scale_log2 - m) : 0.f;
-          l += p0 + p1;
-          __nv_bfloat162 t = __floats2bfloat162_rn(p0, p1);
-          pk[e >> 1] = *reinterpret_cast<uint32_t*>(&t);
-        }
-        // keys c*32 .. c*32+31: box (c >> 1), 16-byte chunks 4*(c & 1) .. +3
-        uint8_t* rowp = sP + (c >> 1) * C::BOX + r * 128;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int chunk = 4 * (c & 1) + k;
-          *reinterpret_cast<uint4*>(rowp + ((chunk ^ (r & 7)) << 4)) =
-              make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
-        }
-      }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      tc_fence_before();
-      mbar_arrive(&p_ready[j & 1]);
-    }
-    if (ok) {
-      int w = 1;
-      if (lane == 0) w = wait_a(o_done, (nkv - 1) & 1, abort_flag) ? 1 : 0;
-      if (__shfl_sync(0xffffffffu, w, 0)) {
-        tc_fence_after();
-        const float inv = 1.0f / l;
-        bf16* orow = reinterpret_cast<bf16*>(a.out) + (size_t)(qs.row0 + r) * a.ld_out + (size_t)h * D;
+      const float alpha = grow ? ex2(m - m_new) : 1.0f;
+      // O_i holds every update through tile j - 1: s_full[i] for tile j
+      // arrived after them
+      if (j >= 1 && __any_sync(0xffffffffu, grow)) {
 #pragma unroll
         for (int c = 0; c < C::DK / 16; ++c) {
           float o[16];
-          tmem_ld16(lane_base + C::TMEM_O + (uint32_t)(c * 16), o);
+          tmem_ld16(o_col + (uint32_t)(c * 16), o);
+#pragma unroll
+          for (int e = 0; e < 16; ++e) o[e] *= alpha;
+          tmem_st16(o_col + (uint32_t)(c * 16), o);
+        }
+      }
+      m = m_use;
+      float ls[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) ls[e] = 0.f;
+      // P as bf16 pairs into the first 64 columns of S_i (already read)
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const float p0 = ex2(fmaf(v[half * 64 + 2 * e], scale_log2, -m));
+          const float p1 = ex2(fmaf(v[half * 64 + 2 * e + 1], scale_log2, -m));
+          ls[e & 7] += p0 + p1;
+          __nv_bfloat162 t2 = __floats2bfloat162_rn(p0, p1);
+          pk[e] = *reinterpret_cast<uint32_t*>(&t2);
+        }
+        tmem_st32(s_col + (uint32_t)(half * 32), pk);
+      }
+      l = l * alpha + (((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7])));
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(&p_ready[i]);
+    }
+    if (ok) {
+      int w = 1;
+      if (lane == 0) w = wait_a(o_final, 0, abort_flag) ? 1 : 0;
+      if (__shfl_sync(0xffffffffu, w, 0)) {
+        tc_fence_after();
+        const float inv = 1.0f / l;
+        bf16* orow = reinterpret_cast<bf16*>(a.out) + (size_t)(qs.row0 + (r < qs.valid ? r : 0)) * a.ld_out + (size_t)h * D;
+#pragma unroll
+        for (int c = 0; c < C::DK / 16; ++c) {
+          float o[16];
+          tmem_ld16(o_col + (uint32_t)(c * 16), o);
           if (r < qs.valid) {
 #pragma unroll
             for (int e = 0; e < 16; e += 8) {
               if (c * 16 + e < D) {
-                float t[8];
+                float t8[8];
 #pragma unroll
-                for (int z = 0; z < 8; ++z) t[z] = o[e + z] * inv;
-                st16(orow + c * 16 + e, t);
+                for (int z = 0; z < 8; ++z) t8[z] = o[e + z] * inv;
+                st16(orow + c * 16 + e, t8);
               }
             }
           }
@@ -338,7 +436,8 @@ cudaError_t attn_tc_t(const AttnArgs& a, cudaStream_t s) {
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  dim3 grid((a.Nt + 127) / 128 + (a.Ni + 127) / 128, a.H, a.B);
+  const int nq = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;  // query tiles per sample, two per CTA
+  dim3 grid((nq + 1) / 2, a.H, a.B);
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)D);
   k_attn_tc<D><<<grid, ATHREADS, ACfg<D>::SMEM, s>>>(tm, a, scale_log2);
   return launched();

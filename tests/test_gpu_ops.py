@@ -203,8 +203,8 @@ ATTN_CASES = [
     ("bf16", 1, 0, 200, 4, 32),
     ("f32", 1, 0, 64, 4, 32),
     ("f32", 2, 7, 40, 2, 72),
-    # from 1024 tokens on the tcgen05 kernel runs: ragged text / image tails,
-    # several query and key tiles, the three head widths it supports
+    # longer sequences: ragged text / image tails, several query and key
+    # tiles (an odd number of query tiles), the tensor-core head widths
     ("bf16", 2, 77, 1000, 2, 128),
     ("bf16", 1, 0, 1100, 3, 72),
     ("bf16", 2, 130, 1030, 2, 64),
