@@ -13,6 +13,14 @@
 // Two TMEM accumulators (2 * BN columns) let the epilogue of tile i overlap
 // the main loop of tile i + 1.  Every mbarrier wait is bounded: on timeout
 // the CTA raises a watchdog flag, stops issuing work and releases its TMEM.
+//
+// A 128 x 128 x 16 MMA takes about as long as a 128 x 256 x 16 one, so
+// narrow tiles run at half rate.  With BN = 256 the columns past the last
+// full 256-wide tile are covered by swapped tiles: up to 128 rows of W as
+// the MMA's M side against 256 rows of A as its N side (the accumulator
+// holds the transposed block; the epilogue transposes it back through a
+// 16 x 32 shared-memory buffer per warp).  DiT-XL/2's N = 1152 layers then
+// run as 4 x 32 full tiles + 16 swapped tiles, one wave of 144 tiles.
 #include "ff_common.cuh"
 #include "ff_tc.cuh"
 
@@ -42,23 +50,47 @@ template <int BN> struct Cfg {
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + 256;
+  // swapped tiles (BN = 256 only): a 16 x 32 fp32 transpose buffer per epilogue warp
+  static constexpr uint32_t XPOSE_BYTES = BN >= 256 ? 8 * 16 * 32 * 4 : 0;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + XPOSE_BYTES + 256;
   // instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
   // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                                     ((uint32_t)(BM >> 4) << 24);
 };
 
+// Tile list of one launch: n_norm normal tiles (128 rows of A x BN rows of
+// W, M-fastest), then swapped tiles (128 rows of W x 256 rows of A).
+struct TileMap {
+  int num_m;   // 128-row blocks of A
+  int n_full;  // BN-wide column blocks of the normal tiles
+  int n_norm;  // num_m * n_full
+  int num_m2;  // 256-row blocks of A (swapped tiles)
+  int n_tiles; // n_norm + swapped tiles
+};
+struct TileAt {
+  bool sw;
+  int m0, n0;  // first output row / column
+};
+template <int BN>
+__device__ __forceinline__ TileAt tile_at(const TileMap& t, int tile) {
+  if (tile < t.n_norm) return {false, (tile % t.num_m) * BM, (tile / t.num_m) * BN};
+  const int u = tile - t.n_norm;
+  return {true, (u % t.num_m2) * 256, t.n_full * BN + (u / t.num_m2) * 128};
+}
+
 template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
-    k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
-              EpiArgs e) {
+    k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+              const __grid_constant__ CUtensorMap tmW128, const __grid_constant__ CUtensorMap tmA256, int M, int N,
+              int K, TileMap tm, EpiArgs e) {
   using C = Cfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
+  float* xpose = reinterpret_cast<float*>(sB + C::STAGES * C::B_BYTES);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES + C::XPOSE_BYTES);
   uint64_t* empty = full + C::STAGES;
   uint64_t* tfull = empty + C::STAGES;
   uint64_t* tempty = tfull + 2;
@@ -66,8 +98,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int num_m = (M + BM - 1) / BM, num_n = (N + BN - 1) / BN;
-  const int num_tiles = num_m * num_n;
+  const int num_tiles = tm.n_tiles;
   const int num_kb = (K + BK - 1) / BK;
 
   if (threadIdx.x == 0) {
@@ -83,6 +114,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
+    if (tm.n_tiles > tm.n_norm) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmW128) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA256) : "memory");
+    }
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(tmem_slot)),
@@ -100,14 +135,22 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-        const int mb = tile % num_m, nb = tile / num_m;
+        const TileAt t = tile_at<BN>(tm, tile);
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
           if (!mbar_wait_g(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
           mbar_expect_tx(&full[s], C::STAGE_BYTES);
-          tma_load(&tmA, &full[s], sA + s * C::A_BYTES, kb * BK, mb * BM);
-          tma_load(&tmB, &full[s], sB + s * C::B_BYTES, kb * BK, nb * BN);
+          // normal: A rows -> M side, W rows -> N side; swapped: the reverse.
+          // (Each call names its kernel parameter: a tensor map must stay in
+          // parameter space, never be copied to local memory.)
+          if (!t.sw) {
+            tma_load(&tmA, &full[s], sA + s * C::A_BYTES, kb * BK, t.m0);
+            tma_load(&tmB, &full[s], sB + s * C::B_BYTES, kb * BK, t.n0);
+          } else {
+            tma_load(&tmW128, &full[s], sA + s * C::A_BYTES, kb * BK, t.n0);
+            tma_load(&tmA256, &full[s], sB + s * C::B_BYTES, kb * BK, t.m0);
+          }
         }
       }
       // Copies still in flight complete on their full barriers; wait for
@@ -156,8 +199,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int h = (warp - 2) >> 2;
     const int row = q * 32 + lane;
     int tc = 0;
+    float* xp = xpose + (warp - 2) * 16 * 32;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++tc) {
-      const int mb = tile % num_m, nb = tile / num_m;
+      const TileAt t = tile_at<BN>(tm, tile);
       const int acc = tc & 1;
       const uint32_t aph = (tc >> 1) & 1;
       int ok = 1;
@@ -165,13 +209,39 @@ __global__ void __launch_bounds__(THREADS, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
-      const int m = mb * BM + row;
-      for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
-        const int n0 = nb * BN + c;
-        if (n0 >= N) break;
-        float v[32];
-        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN + c), v);
-        if (m < M) epi_chunk<bf16, 32>(e, m, n0, N, v);
+      const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+      if (!t.sw) {
+        const int m = t.m0 + row;
+        for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
+          const int n0 = t.n0 + c;
+          if (n0 >= N) break;
+          float v[32];
+          tmem_ld32(tq + (uint32_t)c, v);
+          if (m < M) epi_chunk<bf16, 32>(e, m, n0, N, v);
+        }
+      } else if constexpr (C::XPOSE_BYTES > 0) {
+        // lane = output column n + lane; TMEM column = output row.  Blocks of
+        // 16 rows x 32 columns go through the warp's buffer (XOR-swizzled,
+        // conflict-free both ways); afterwards lane l holds row l / 2,
+        // columns 16 (l % 2) .. + 15.
+        const int n = t.n0 + q * 32;
+        for (int c = h * (BN / 2); c < (h + 1) * (BN / 2) && n < N; c += 16) {
+          const int m0 = t.m0 + c;
+          if (m0 >= M) break;
+          {
+            float u[16];
+            tmem_ld16(tq + (uint32_t)c, u);  // u[j] = out[m0 + j][n + lane]
+#pragma unroll
+            for (int j = 0; j < 16; ++j) xp[j * 32 + (lane ^ j)] = u[j];
+          }
+          __syncwarp();
+          const int r = lane >> 1, c0 = (lane & 1) * 16;
+          float v[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) v[j] = xp[r * 32 + ((c0 + j) ^ r)];  // out[m0 + r][n + c0 + j]
+          __syncwarp();
+          if (m0 + r < M) epi_chunk<bf16, 16>(e, m0 + r, n + c0, N, v);
+        }
       }
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
@@ -441,14 +511,34 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
       k_gemm_tc2<128><<<grid, THREADS, Cfg2<128>::SMEM, s>>>(ma, mb, M, N, K, e);
     return launched();
   }
-  const int bn = pick_bn(M, N, BM, g_sms);
-  if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, bn)) return cudaErrorInvalidValue;
-  const long long tiles = (long long)((M + BM - 1) / BM) * ((N + bn - 1) / bn);
-  const int grid = (int)(tiles < g_sms ? tiles : g_sms);
-  if (bn == 256)
-    k_gemm_tc<256><<<grid, THREADS, Cfg<256>::SMEM, s>>>(ma, mb, M, N, K, e);
-  else
-    k_gemm_tc<128><<<grid, THREADS, Cfg<128>::SMEM, s>>>(ma, mb, M, N, K, e);
+  // Every tile (128 x 256 full rate, 128 x 128 at half rate, swapped 128 x
+  // 256) takes about the same time: take the tiling with the fewest waves,
+  // ties to full-rate tiles.
+  TileMap tm;
+  tm.num_m = (M + BM - 1) / BM;
+  tm.num_m2 = (M + 255) / 256;
+  const int rem = N % 256;
+  const long long t256 = (long long)tm.num_m * (N / 256) + (rem ? (long long)((rem + 127) / 128) * tm.num_m2 : 0);
+  const long long t128 = (long long)tm.num_m * ((N + 127) / 128);
+  const bool wide = (t256 + g_sms - 1) / g_sms <= (t128 + g_sms - 1) / g_sms;
+  CUtensorMap mw128 = {}, ma256 = {};
+  if (wide) {
+    tm.n_full = N / 256;
+    tm.n_norm = tm.num_m * tm.n_full;
+    tm.n_tiles = (int)t256;
+    if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, 256)) return cudaErrorInvalidValue;
+    if (rem && (!make_map(&mw128, W, N, K, ldw, BM) || !make_map(&ma256, A, M, K, lda, 256)))
+      return cudaErrorInvalidValue;
+    const int grid = (int)(t256 < g_sms ? t256 : g_sms);
+    k_gemm_tc<256><<<grid, THREADS, Cfg<256>::SMEM, s>>>(ma, mb, mw128, ma256, M, N, K, tm, e);
+  } else {
+    tm.n_full = (N + 127) / 128;
+    tm.n_norm = tm.num_m * tm.n_full;
+    tm.n_tiles = tm.n_norm;
+    if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, 128)) return cudaErrorInvalidValue;
+    const int grid = (int)(t128 < g_sms ? t128 : g_sms);
+    k_gemm_tc<128><<<grid, THREADS, Cfg<128>::SMEM, s>>>(ma, mb, ma, mb, M, N, K, tm, e);
+  }
   return launched();
 }
 
