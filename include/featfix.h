@@ -81,6 +81,16 @@ enum { FEATFIX_PLAN_EXACT = 0, FEATFIX_PLAN_DRAFT = 1, FEATFIX_PLAN_SITE = 2 };
  * sites) and the paid check runs on a shadow copy that chains the per-block
  * drafts up to the site.  Steps with a debug capture always run per block. */
 #define FEATFIX_FLAG_PER_BLOCK_DRAFT 2u
+/* SITE_UPDATES_HISTORY takes the other reading of where the finite
+ * differences of Eq. 2 are estimated: a site's exact increment h^f - u
+ * (Eq. 3) is pushed onto its block's history like a refresh, after the
+ * site's own draft (and its discrepancy, Eq. 4) used the history before
+ * it.  Later drafts of that block then interpolate its own refresh-and-site
+ * steps (featfix_plan_build_blocks gives the per-block weights).  Default
+ * off: sites leave the history alone, so the draft policy outside the site
+ * set is the base policy's and Verify and FeatFix share their caches.
+ * Drafted steps then run per block (no telescoping).                       */
+#define FEATFIX_FLAG_SITE_UPDATES_HISTORY 4u
 
 /*
  * Model shape (Eq. 1's block B_l and the surrounding sampler).
@@ -246,6 +256,14 @@ FEATFIX_API featfix_status featfix_plan_build(int steps, int n_layers, const int
                                   int draft_order, const featfix_site* sites, int n_sites,
                                   int mode, unsigned flags, unsigned char* kinds, int* k_eff,
                                   double* weights);
+
+/* Host-only: per (step, block) draft order k_eff [steps*n_layers] (-1
+ * where the block is exact) and weights [steps*n_layers*4] of the history
+ * that block's draft reads.  Equal to featfix_plan_build's per-step values
+ * for every block unless flags has FEATFIX_FLAG_SITE_UPDATES_HISTORY.        */
+FEATFIX_API featfix_status featfix_plan_build_blocks(int steps, int n_layers, const int* refresh, int n_refresh,
+                                         int draft_order, const featfix_site* sites, int n_sites, int mode,
+                                         unsigned flags, int* k_eff, double* weights);
 
 /* Debug capture: during later trajectories, copy block `layer`'s incoming
  * state u and its forwarded output at step `step` into dev_in / dev_out

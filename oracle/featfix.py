@@ -9,8 +9,11 @@ Per denoising step i the L blocks run in order on the incoming state u:
   the discrepancy ||h_d - h_f||_1 / (||h_f||_1 + eps) (Eq. 4) and its L2
   analogue are logged and never route the sample; the forwarded output is
   h_f for FeatFix (Eq. 5) and h_d for Verify.  Exact-only drops the draft and
-  the discrepancy and forwards h_f.  A site's exact output does not enter the
-  refresh history, so the draft policy outside S is the base policy's.
+  the discrepancy and forwards h_f.  By default a site's exact output does
+  not enter the refresh history, so the draft policy outside S is the base
+  policy's; with ``site_updates_history`` (the alternative reading of where
+  the paper's differences are estimated) the site's increment h_f - u is
+  pushed onto block l's history like a refresh, after its own draft.
 * Vanilla: every block exact, no history.
 
 Accounting (Section 3.3): full-refresh steps, paid checks and forwarded
@@ -49,7 +52,7 @@ def model_input(shape, x):
 
 
 def run(W, shape, cond, x_T, steps, refresh, K, sites, mode="featfix",
-        variant="interp", hook=None):
+        variant="interp", hook=None, site_updates_history=False):
     """Run the cached sampler.
 
     W      dict of float64 weights.
@@ -57,6 +60,8 @@ def run(W, shape, cond, x_T, steps, refresh, K, sites, mode="featfix",
     x_T    initial latent [B_lat, ...].
     sites  (step, layer) pairs.
     hook   optional callable(step, layer, kind, u, h_out, extra) for tests.
+    site_updates_history   push a site's exact increment onto its block's
+           history (after the site's own draft).
 
     Returns (x_0, logs, counters) with logs = list of dicts
     {step, layer, rel_l1, rel_l2} in execution order and counters =
@@ -105,6 +110,9 @@ def run(W, shape, cond, x_T, steps, refresh, K, sites, mode="featfix",
                     else:
                         h = hd
                     extra = {"h_d": hd, "h_f": hf}
+                if site_updates_history:
+                    hist[l].insert(0, (i, hf - u))
+                    del hist[l][K + 1:]
             if hook is not None:
                 hook(i, l, k, u, h, extra)
             tok = h

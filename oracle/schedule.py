@@ -51,6 +51,29 @@ def validate(steps, L, refresh, K, sites):
         seen.add((i, l))
 
 
+def block_history_steps(steps, L, refresh, K, sites, mode, site_updates_history=False):
+    """Per (step, layer) the steps of the history entries a draft at that
+    point reads, newest first (at most K + 1), or None where no draft is
+    formed (exact blocks, the vanilla arm).  Refreshes push every block; with
+    ``site_updates_history`` a site pushes its own block after its draft."""
+    kind, _ = build_plan(steps, L, refresh, K, sites, mode)
+    nodes = [[] for _ in range(L)]
+    out = []
+    for i in range(steps):
+        row = []
+        for l in range(L):
+            if kind[i][l] == EXACT:
+                row.append(None)
+                if mode != "vanilla":
+                    nodes[l] = ([i] + nodes[l])[:K + 1]
+            else:
+                row.append(list(nodes[l]))
+                if kind[i][l] == SITE and site_updates_history:
+                    nodes[l] = ([i] + nodes[l])[:K + 1]
+        out.append(row)
+    return out
+
+
 def build_plan(steps, L, refresh, K, sites, mode):
     """Return (kind[steps][L], k_eff[steps]).
 

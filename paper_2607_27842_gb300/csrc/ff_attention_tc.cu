@@ -44,8 +44,10 @@ constexpr size_t SMEM_LIMIT = 232448;  // opt-in dynamic shared memory per block
 
 __device__ unsigned int g_attn_watchdog;
 
+// Every hand-off in this kernel (S ready -> softmax -> P ready -> MMA) is on
+// the critical path, so waits poll instead of suspending.
 __device__ __forceinline__ bool wait_a(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
-  return mbar_wait(b, parity, abort_flag, &g_attn_watchdog);
+  return mbar_wait<true>(b, parity, abort_flag, &g_attn_watchdog);
 }
 
 template <int D> struct ACfg {
@@ -198,6 +200,10 @@ __global__ void __launch_bounds__(ATHREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // dependents may launch once every CTA holds its TMEM; the previous
+  // kernel's outputs are complete after the wait
+  pdl_trigger();
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -439,7 +445,7 @@ cudaError_t attn_tc_t(const AttnArgs& a, cudaStream_t s) {
   const int nq = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;  // query tiles per sample, two per CTA
   dim3 grid((nq + 1) / 2, a.H, a.B);
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)D);
-  k_attn_tc<D><<<grid, ATHREADS, ACfg<D>::SMEM, s>>>(tm, a, scale_log2);
+  launch_pdl(k_attn_tc<D>, grid, ATHREADS, ACfg<D>::SMEM, s, tm, a, scale_log2);
   return launched();
 }
 

@@ -110,25 +110,9 @@ __device__ __forceinline__ int epi_batch(const EpiArgs& e, int r) {
   return r < e.seg_split ? r / e.rpb0 : (r - e.seg_split) / e.rpb1;
 }
 
-// Applies the epilogue to CH consecutive accumulator columns n0 .. n0+CH-1
-// of row m.  The chunk must not straddle split_col, act_col0 or rope_cols,
-// and CH must be a multiple of the 16-byte vector width of T.  Columns >= N
-// are skipped (N % vector width == 0).
+// RoPE on q / k columns of image rows, then the activation.
 template <class T, int CH>
-__device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N, float (&v)[CH]) {
-  constexpr int V = VecN<T>::n;
-  if (e.bias) {
-    const T* b = reinterpret_cast<const T*>(e.bias);
-#pragma unroll
-    for (int j = 0; j < CH; j += V) {
-      if (n0 + j < N) {
-        float bb[V];
-        ld16(b + n0 + j, bb);
-#pragma unroll
-        for (int q = 0; q < V; ++q) v[j + q] += bb[q];
-      }
-    }
-  }
+__device__ __forceinline__ void epi_rope_act(const EpiArgs& e, int m, int n0, float (&v)[CH]) {
   if (e.rope && m >= e.rope_row0 && n0 < e.rope_cols) {
     const int tok = (m - e.rope_row0) % e.rope_period;
     const int half = e.rope_hd >> 1;
@@ -148,6 +132,30 @@ __device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N
 #pragma unroll
     for (int j = 0; j < CH; ++j) v[j] = silu(v[j]);
   }
+}
+
+// Applies the epilogue to CH consecutive accumulator columns n0 .. n0+CH-1
+// of row m.  The chunk must not straddle split_col, act_col0 or rope_cols,
+// and CH must be a multiple of the 16-byte vector width of T.  Columns >= N
+// are skipped (N % vector width == 0).
+// The part of the epilogue before the residual: y = gate * act(acc + bias),
+// with RoPE applied to q / k columns.
+template <class T, int CH>
+__device__ __forceinline__ void epi_math(const EpiArgs& e, int m, int n0, int N, float (&v)[CH]) {
+  constexpr int V = VecN<T>::n;
+  if (e.bias) {
+    const T* b = reinterpret_cast<const T*>(e.bias);
+#pragma unroll
+    for (int j = 0; j < CH; j += V) {
+      if (n0 + j < N) {
+        float bb[V];
+        ld16(b + n0 + j, bb);
+#pragma unroll
+        for (int q = 0; q < V; ++q) v[j + q] += bb[q];
+      }
+    }
+  }
+  epi_rope_act<T, CH>(e, m, n0, v);
   if (e.gate) {
     const float* g = e.gate + (size_t)epi_batch(e, m) * e.gate_stride + n0;
 #pragma unroll
@@ -158,6 +166,12 @@ __device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N
       }
     }
   }
+}
+
+template <class T, int CH>
+__device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N, float (&v)[CH]) {
+  constexpr int V = VecN<T>::n;
+  epi_math<T, CH>(e, m, n0, N, v);
   if (e.resid) {
     const T* rs = reinterpret_cast<const T*>(e.resid) + (size_t)m * e.ld_resid + n0;
 #pragma unroll
@@ -209,6 +223,32 @@ __device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N
       }
     }
   }
+}
+
+// ---------------------------------------------------------------------------
+// programmatic dependent launch: a kernel launched with launch_pdl may start
+// while the previous kernel on the stream is still finishing.  It lets its
+// own dependents launch (pdl_trigger) and then waits for the previous
+// kernel to complete, memory included (pdl_wait), before it touches global
+// memory.  Both are no-ops in a kernel launched the ordinary way.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+static inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                                     Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
 // ---------------------------------------------------------------------------

@@ -57,6 +57,8 @@ __device__ __forceinline__ float draft_scalar(const T* xu, const Hist4& h, const
 template <class T, int NT>
 __global__ void __launch_bounds__(256) k_draft(T* __restrict__ x, Hist4 h, float w0, float w1, float w2, float w3,
                                                long long n) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int V = VecN<T>::n;
   const float w[4] = {w0, w1, w2, w3};
   const long long nvec = n / V;
@@ -85,10 +87,10 @@ static cudaError_t draft_t(void* x, const Hist4& h, const float* w, int nt, long
   const int grid = stream_grid(n / VecN<T>::n, 256);
   T* xp = reinterpret_cast<T*>(x);
   switch (nt) {
-    case 1: k_draft<T, 1><<<grid, 256, 0, s>>>(xp, h, w[0], w[1], w[2], w[3], n); break;
-    case 2: k_draft<T, 2><<<grid, 256, 0, s>>>(xp, h, w[0], w[1], w[2], w[3], n); break;
-    case 3: k_draft<T, 3><<<grid, 256, 0, s>>>(xp, h, w[0], w[1], w[2], w[3], n); break;
-    case 4: k_draft<T, 4><<<grid, 256, 0, s>>>(xp, h, w[0], w[1], w[2], w[3], n); break;
+    case 1: launch_pdl(k_draft<T, 1>, grid, 256, 0, s, xp, h, w[0], w[1], w[2], w[3], n); break;
+    case 2: launch_pdl(k_draft<T, 2>, grid, 256, 0, s, xp, h, w[0], w[1], w[2], w[3], n); break;
+    case 3: launch_pdl(k_draft<T, 3>, grid, 256, 0, s, xp, h, w[0], w[1], w[2], w[3], n); break;
+    case 4: launch_pdl(k_draft<T, 4>, grid, 256, 0, s, xp, h, w[0], w[1], w[2], w[3], n); break;
     default: return cudaErrorInvalidValue;
   }
   return launched();
@@ -103,6 +105,8 @@ cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int 
 template <class T>
 __global__ void __launch_bounds__(256) k_diff(const T* __restrict__ a, const T* __restrict__ b, T* __restrict__ out,
                                               long long n) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int V = VecN<T>::n;
   const long long nvec = n / V;
   const long long stride = (long long)gridDim.x * blockDim.x;
@@ -123,9 +127,9 @@ __global__ void __launch_bounds__(256) k_diff(const T* __restrict__ a, const T* 
 cudaError_t launch_diff(DType dt, const void* a, const void* b, void* out, long long n, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   if (dt == F32) {
-    k_diff<float><<<stream_grid(n / 4, 256), 256, 0, s>>>((const float*)a, (const float*)b, (float*)out, n);
+    launch_pdl(k_diff<float>, stream_grid(n / 4, 256), 256, 0, s, (const float*)a, (const float*)b, (float*)out, n);
   } else {
-    k_diff<bf16><<<stream_grid(n / 8, 256), 256, 0, s>>>((const bf16*)a, (const bf16*)b, (bf16*)out, n);
+    launch_pdl(k_diff<bf16>, stream_grid(n / 8, 256), 256, 0, s, (const bf16*)a, (const bf16*)b, (bf16*)out, n);
   }
   return launched();
 }
@@ -166,6 +170,8 @@ template <class T, int NT>
 __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_THREADS)
     k_verify(T* __restrict__ u, Hist4 h, float w0, float w1, float w2, float w3, const T* __restrict__ hf,
              long long n, int write_draft, double* __restrict__ partials) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int V = VecN<T>::n;
   const float w[4] = {w0, w1, w2, w3};
   float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
@@ -219,6 +225,8 @@ __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_
 }
 
 __global__ void k_verify_finish(const double* __restrict__ partials, int nparts, double* __restrict__ sums) {
+  pdl_trigger();
+  pdl_wait();
   if (threadIdx.x < 4) {
     double t = 0.0;
     for (int k = 0; k < nparts; ++k) t += partials[(size_t)k * 4 + threadIdx.x];
@@ -234,15 +242,15 @@ static cudaError_t verify_t(void* u, const Hist4& h, const float* w, int nt, con
   T* up = reinterpret_cast<T*>(u);
   const T* fp = reinterpret_cast<const T*>(hf);
   switch (nt) {
-    case 1: k_verify<T, 1><<<grid, VERIFY_THREADS, 0, s>>>(up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
-    case 2: k_verify<T, 2><<<grid, VERIFY_THREADS, 0, s>>>(up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
-    case 3: k_verify<T, 3><<<grid, VERIFY_THREADS, 0, s>>>(up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
-    case 4: k_verify<T, 4><<<grid, VERIFY_THREADS, 0, s>>>(up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    case 1: launch_pdl(k_verify<T, 1>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    case 2: launch_pdl(k_verify<T, 2>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    case 3: launch_pdl(k_verify<T, 3>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    case 4: launch_pdl(k_verify<T, 4>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
     default: return cudaErrorInvalidValue;
   }
   cudaError_t e = launched();
   if (e != cudaSuccess) return e;
-  k_verify_finish<<<1, 32, 0, s>>>(parts, grid / VERIFY_CLUSTER, sums);
+  launch_pdl(k_verify_finish, 1, 32, 0, s, parts, grid / VERIFY_CLUSTER, sums);
   return launched();
 }
 
@@ -262,6 +270,8 @@ template <class T, int NCH>
 __global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
                                                 const float* __restrict__ shift, const float* __restrict__ scale,
                                                 int mod_stride, int seg_split, int rpb0, int rpb1) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int V = VecN<T>::n;
   const long long r = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -323,14 +333,14 @@ static cudaError_t ln_mod_t(const void* x, void* out, long long rows, int C, con
   const T* xp = (const T*)x;
   T* op = (T*)out;
 #define FF_LN_CASE(n) \
-  case n: k_ln_mod<T, n><<<grid, 256, 0, s>>>(xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break;
+  case n: launch_pdl(k_ln_mod<T, n>, grid, 256, 0, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break;
   switch (nch) {
     FF_LN_CASE(1) FF_LN_CASE(2) FF_LN_CASE(3) FF_LN_CASE(4) FF_LN_CASE(5) FF_LN_CASE(6)
     FF_LN_CASE(8) FF_LN_CASE(12) FF_LN_CASE(16)
     default:
-      if (nch <= 8) { k_ln_mod<T, 8><<<grid, 256, 0, s>>>(xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
-      if (nch <= 12) { k_ln_mod<T, 12><<<grid, 256, 0, s>>>(xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
-      if (nch <= 16) { k_ln_mod<T, 16><<<grid, 256, 0, s>>>(xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      if (nch <= 8) { launch_pdl(k_ln_mod<T, 8>, grid, 256, 0, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      if (nch <= 12) { launch_pdl(k_ln_mod<T, 12>, grid, 256, 0, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      if (nch <= 16) { launch_pdl(k_ln_mod<T, 16>, grid, 256, 0, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
       return cudaErrorInvalidValue;
   }
 #undef FF_LN_CASE
@@ -348,6 +358,8 @@ cudaError_t launch_ln_mod(DType dt, const void* x, void* out, long long rows, in
 // Sinusoidal features of every model time: row s = [cos(t_s f_k) | sin(t_s f_k)].
 template <class T>
 __global__ void k_sinusoid_table(const float* __restrict__ times, int S, T* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   const int s = blockIdx.x;
   if (s >= S) return;
   const double t = (double)times[s];
@@ -360,8 +372,8 @@ __global__ void k_sinusoid_table(const float* __restrict__ times, int S, T* __re
 
 cudaError_t launch_sinusoid_table(DType dt, const float* times, int S, void* out, cudaStream_t s) {
   if (S <= 0) return cudaSuccess;
-  if (dt == F32) k_sinusoid_table<float><<<S, 128, 0, s>>>(times, S, (float*)out);
-  else k_sinusoid_table<bf16><<<S, 128, 0, s>>>(times, S, (bf16*)out);
+  if (dt == F32) launch_pdl(k_sinusoid_table<float>, S, 128, 0, s, times, S, (float*)out);
+  else launch_pdl(k_sinusoid_table<bf16>, S, 128, 0, s, times, S, (bf16*)out);
   return launched();
 }
 
@@ -370,6 +382,8 @@ template <class T>
 __global__ void k_cond_table(const float* __restrict__ temb, const T* __restrict__ y_emb, const int* __restrict__ labels,
                              int S, int B, int C, const int* __restrict__ need_row, T* __restrict__ all,
                              T* __restrict__ need) {
+  pdl_trigger();
+  pdl_wait();
   const int row = blockIdx.x;  // s * B + b
   const int s = row / B, b = row % B;
   if (s >= S) return;
@@ -387,10 +401,10 @@ cudaError_t launch_cond_table(DType dt, const float* temb, const void* y_emb, co
                               const int* need_row, void* all, void* need, cudaStream_t s) {
   if (S <= 0) return cudaSuccess;
   if (dt == F32)
-    k_cond_table<float><<<S * B, 256, 0, s>>>(temb, (const float*)y_emb, labels, S, B, C, need_row, (float*)all,
+    launch_pdl(k_cond_table<float>, S * B, 256, 0, s, temb, (const float*)y_emb, labels, S, B, C, need_row, (float*)all,
                                               (float*)need);
   else
-    k_cond_table<bf16><<<S * B, 256, 0, s>>>(temb, (const bf16*)y_emb, labels, S, B, C, need_row, (bf16*)all,
+    launch_pdl(k_cond_table<bf16>, S * B, 256, 0, s, temb, (const bf16*)y_emb, labels, S, B, C, need_row, (bf16*)all,
                                              (bf16*)need);
   return launched();
 }
@@ -400,6 +414,8 @@ cudaError_t launch_cond_table(DType dt, const float* temb, const void* y_emb, co
 template <class T>
 __global__ void k_patchify(const float* __restrict__ lat, int B_lat, int B_model, int Cin, int F, int H, int W, int p,
                            int pt, T* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   const int Ff = F > 0 ? F : 1, ptt = F > 0 ? pt : 1;
   const int gf = Ff / ptt, gh = H / p, gw = W / p;
   const int P = ptt * p * p, feat = Cin * P;
@@ -421,13 +437,15 @@ __global__ void k_patchify(const float* __restrict__ lat, int B_lat, int B_model
 cudaError_t launch_patchify(DType dt, const float* latent, int B_lat, int B_model, int Cin, int F, int H, int W,
                             int p, int pt, void* out, cudaStream_t s) {
   const int grid = num_sms() * 4;
-  if (dt == F32) k_patchify<float><<<grid, 256, 0, s>>>(latent, B_lat, B_model, Cin, F, H, W, p, pt, (float*)out);
-  else k_patchify<bf16><<<grid, 256, 0, s>>>(latent, B_lat, B_model, Cin, F, H, W, p, pt, (bf16*)out);
+  if (dt == F32) launch_pdl(k_patchify<float>, grid, 256, 0, s, latent, B_lat, B_model, Cin, F, H, W, p, pt, (float*)out);
+  else launch_pdl(k_patchify<bf16>, grid, 256, 0, s, latent, B_lat, B_model, Cin, F, H, W, p, pt, (bf16*)out);
   return launched();
 }
 
 template <class T>
 __global__ void k_convert(const float* __restrict__ in, T* __restrict__ out, long long n) {
+  pdl_trigger();
+  pdl_wait();
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x)
     out[i] = from_f<T>(in[i]);
 }
@@ -435,8 +453,8 @@ __global__ void k_convert(const float* __restrict__ in, T* __restrict__ out, lon
 cudaError_t launch_convert(DType dt, const float* in, void* out, long long n, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int grid = num_sms() * 4;
-  if (dt == F32) k_convert<float><<<grid, 256, 0, s>>>(in, (float*)out, n);
-  else k_convert<bf16><<<grid, 256, 0, s>>>(in, (bf16*)out, n);
+  if (dt == F32) launch_pdl(k_convert<float>, grid, 256, 0, s, in, (float*)out, n);
+  else launch_pdl(k_convert<bf16>, grid, 256, 0, s, in, (bf16*)out, n);
   return launched();
 }
 
@@ -446,6 +464,8 @@ cudaError_t launch_convert(DType dt, const float* in, void* out, long long n, cu
 // c1 = sqrt(a_prev / a_t), c2 = sqrt(1 - a_prev) - sqrt(a_prev (1 - a_t) / a_t).
 __global__ void k_sampler(const float* __restrict__ mo, float* __restrict__ lat, int B_lat, int cfg, float cfg_scale,
                           int Cin, int Cout, int F, int H, int W, int p, int pt, float c1, float c2) {
+  pdl_trigger();
+  pdl_wait();
   const int Ff = F > 0 ? F : 1, ptt = F > 0 ? pt : 1;
   const int gh = H / p, gw = W / p, gf = Ff / ptt;
   const int P = ptt * p * p;
@@ -471,7 +491,7 @@ __global__ void k_sampler(const float* __restrict__ mo, float* __restrict__ lat,
 
 cudaError_t launch_sampler(const float* model_out, float* latent, int B_lat, int cfg, float cfg_scale, int Cin,
                            int Cout, int F, int H, int W, int p, int pt, float c1, float c2, cudaStream_t s) {
-  k_sampler<<<num_sms() * 2, 256, 0, s>>>(model_out, latent, B_lat, cfg, cfg_scale, Cin, Cout, F, H, W, p, pt, c1, c2);
+  launch_pdl(k_sampler, num_sms() * 2, 256, 0, s, model_out, latent, B_lat, cfg, cfg_scale, Cin, Cout, F, H, W, p, pt, c1, c2);
   return launched();
 }
 
@@ -485,6 +505,8 @@ __device__ __forceinline__ unsigned long long splitmix_word(unsigned long long s
 }
 
 __global__ void k_noise(unsigned long long seed, float* __restrict__ out, long long n) {
+  pdl_trigger();
+  pdl_wait();
   const long long pairs = (n + 1) / 2;
   for (long long m = (long long)blockIdx.x * blockDim.x + threadIdx.x; m < pairs; m += (long long)gridDim.x * blockDim.x) {
     const double u1 = ((double)(splitmix_word(seed, 2 * m) >> 11) + 0.5) * 0x1.0p-53;
@@ -498,7 +520,7 @@ __global__ void k_noise(unsigned long long seed, float* __restrict__ out, long l
 }
 
 cudaError_t launch_noise(unsigned long long seed, float* out, long long n, cudaStream_t s) {
-  k_noise<<<num_sms() * 2, 256, 0, s>>>(seed, out, n);
+  launch_pdl(k_noise, num_sms() * 2, 256, 0, s, seed, out, n);
   return launched();
 }
 
@@ -507,6 +529,8 @@ cudaError_t launch_noise(unsigned long long seed, float* out, long long n, cudaS
 // [sin(pos w_k) | cos(pos w_k)], w_k = 10000^(-k/(C/4)).
 template <class T>
 __global__ void k_pos2d(T* __restrict__ out, int B, int gh, int gw, int C) {
+  pdl_trigger();
+  pdl_wait();
   const int q = C / 4;
   const long long total = (long long)B * gh * gw * C;
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long long)gridDim.x * blockDim.x) {
@@ -522,8 +546,8 @@ __global__ void k_pos2d(T* __restrict__ out, int B, int gh, int gw, int C) {
 
 cudaError_t launch_pos2d(DType dt, void* out, int B, int gh, int gw, int C, cudaStream_t s) {
   const int grid = num_sms() * 4;
-  if (dt == F32) k_pos2d<float><<<grid, 256, 0, s>>>((float*)out, B, gh, gw, C);
-  else k_pos2d<bf16><<<grid, 256, 0, s>>>((bf16*)out, B, gh, gw, C);
+  if (dt == F32) launch_pdl(k_pos2d<float>, grid, 256, 0, s, (float*)out, B, gh, gw, C);
+  else launch_pdl(k_pos2d<bf16>, grid, 256, 0, s, (bf16*)out, B, gh, gw, C);
   return launched();
 }
 

@@ -50,8 +50,10 @@ template <int BN> struct Cfg {
   static constexpr uint32_t B_BYTES = BN * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
-  // swapped tiles (BN = 256 only): a 16 x 32 fp32 transpose buffer per epilogue warp
-  static constexpr uint32_t XPOSE_BYTES = BN >= 256 ? 8 * 16 * 32 * 4 : 0;
+  // BN = 256 only: 4 KB per epilogue warp, two 32 x 32 bf16 output blocks
+  // for the TMA-store epilogue, or the 16 x 32 fp32 transpose buffer of a
+  // swapped tile
+  static constexpr uint32_t XPOSE_BYTES = BN >= 256 ? 8 * 4096 : 0;
   static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + XPOSE_BYTES + 256;
   // instruction descriptor, kind::f16: D fp32 (bit 4), A bf16 (bits 7-9 = 1),
   // B bf16 (bits 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
@@ -67,7 +69,18 @@ struct TileMap {
   int n_norm;  // num_m * n_full
   int num_m2;  // 256-row blocks of A (swapped tiles)
   int n_tiles; // n_norm + swapped tiles
+  int staged;  // normal tiles store out (and hist_out) through shared memory + TMA
 };
+
+// 64-byte-swizzled [32 rows x 32 bf16] block: 16-byte chunk k of row r
+__device__ __forceinline__ uint32_t blk_off(int r, int k) { return (uint32_t)(r * 64 + ((k ^ ((r >> 1) & 3)) << 4)); }
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&t);
+}
+__device__ __forceinline__ float2 unpack2(uint32_t u) {
+  return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u));
+}
 struct TileAt {
   bool sw;
   int m0, n0;  // first output row / column
@@ -82,8 +95,9 @@ __device__ __forceinline__ TileAt tile_at(const TileMap& t, int tile) {
 template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-              const __grid_constant__ CUtensorMap tmW128, const __grid_constant__ CUtensorMap tmA256, int M, int N,
-              int K, TileMap tm, EpiArgs e) {
+              const __grid_constant__ CUtensorMap tmW128, const __grid_constant__ CUtensorMap tmA256,
+              const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmH, int M, int N, int K,
+              TileMap tm, EpiArgs e) {
   using C = Cfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -129,6 +143,10 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // dependents may launch once every CTA holds its TMEM; the previous
+  // kernel's outputs are complete after the wait
+  pdl_trigger();
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -199,18 +217,50 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int h = (warp - 2) >> 2;
     const int row = q * 32 + lane;
     int tc = 0;
-    float* xp = xpose + (warp - 2) * 16 * 32;
+    uint8_t* ep = reinterpret_cast<uint8_t*>(xpose) + (warp - 2) * 4096;
+    float* xp = reinterpret_cast<float*>(ep);
+    uint32_t epi_cnt = 0;
+    const int c_lo = h * (BN / 2);
+    uint4 pr[4], ph[4];
+    float pb = 0.f, pg0 = 0.f, pg1 = 0.f;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++tc) {
       const TileAt t = tile_at<BN>(tm, tile);
       const int acc = tc & 1;
       const uint32_t aph = (tc >> 1) & 1;
+      // staged epilogue: residual / history-base rows of chunk n0 into pr /
+      // ph; bias and gate of column n0 + lane into pb / pg0 / pg1 (shared
+      // across the warp by shuffles: the warp's 32 rows lie in samples
+      // b_lo .. b_hi, at most two of them)
+      const int wr0 = t.m0 + q * 32;
+      const int b_lo = e.gate ? epi_batch(e, min(wr0, M - 1)) : 0;
+      const int b_hi = e.gate ? epi_batch(e, min(wr0 + 31, M - 1)) : 0;
+      auto fetch = [&](int n0) {
+        const int m = t.m0 + row;
+        const bool cin = n0 + lane < N;
+        pb = (e.bias && cin) ? __bfloat162float(reinterpret_cast<const bf16*>(e.bias)[n0 + lane]) : 0.f;
+        pg0 = (e.gate && cin) ? e.gate[(size_t)b_lo * e.gate_stride + n0 + lane] : 0.f;
+        pg1 = (e.gate && cin && b_hi != b_lo) ? e.gate[(size_t)b_hi * e.gate_stride + n0 + lane] : pg0;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const bool in = m < M && n0 + 8 * k < N;
+          if (e.resid)
+            pr[k] = in ? *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.resid) +
+                                                          (size_t)m * e.ld_resid + n0 + 8 * k)
+                       : make_uint4(0, 0, 0, 0);
+          if (e.hist_out)
+            ph[k] = in ? *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.hist_base) +
+                                                          (size_t)m * e.ldo + n0 + 8 * k)
+                       : make_uint4(0, 0, 0, 0);
+        }
+      };
+      if (C::XPOSE_BYTES > 0 && tm.staged && !t.sw) fetch(t.n0 + c_lo);
       int ok = 1;
       if (lane == 0) ok = mbar_wait_g(&tfull[acc], aph, abort_flag) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
       const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-      if (!t.sw) {
+      if (!t.sw && (C::XPOSE_BYTES == 0 || !tm.staged)) {
         const int m = t.m0 + row;
         for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
           const int n0 = t.n0 + c;
@@ -219,12 +269,86 @@ __global__ void __launch_bounds__(THREADS, 1)
           tmem_ld32(tq + (uint32_t)c, v);
           if (m < M) epi_chunk<bf16, 32>(e, m, n0, N, v);
         }
+      } else if (!t.sw) {
+        // Staged epilogue: each 32-row x 32-column chunk is written into a
+        // swizzled shared-memory block and stored by one TMA copy (whole
+        // lines instead of one L2 request per 16 bytes).  The residual and
+        // history-base rows of a chunk are loaded ahead: the first chunk's
+        // before the accumulator wait, the next one's while the current
+        // chunk is finished.
+        const int m = t.m0 + row;
+        for (int c = c_lo; c < c_lo + BN / 2; c += 32) {
+          const int n0 = t.n0 + c;
+          if (n0 >= N) break;
+          float v[32];
+          tmem_ld32(tq + (uint32_t)c, v);
+          // y = gate * act(rope(acc + bias)), the order of epi_math; rows
+          // past M are not stored (the TMA store clips them)
+          if (e.bias) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, pb, j);
+          }
+          if (m < M) epi_rope_act<bf16, 32>(e, m, n0, v);
+          if (e.gate) {
+            const bool lo = m >= M || epi_batch(e, m) == b_lo;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              const float g0 = __shfl_sync(0xffffffffu, pg0, j), g1 = __shfl_sync(0xffffffffu, pg1, j);
+              v[j] *= lo ? g0 : g1;
+            }
+          }
+          uint32_t ob[16], hb[16];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const uint32_t rr[4] = {pr[k].x, pr[k].y, pr[k].z, pr[k].w};
+            const uint32_t hh[4] = {ph[k].x, ph[k].y, ph[k].z, ph[k].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              float a = v[8 * k + 2 * i], b = v[8 * k + 2 * i + 1];
+              if (e.resid) {
+                const float2 r2 = unpack2(rr[i]);
+                a += r2.x;
+                b += r2.y;
+              }
+              ob[4 * k + i] = pack2(a, b);
+              if (e.hist_out) {  // stored(out) - hist_base
+                const float2 o2 = unpack2(ob[4 * k + i]), h2 = unpack2(hh[i]);
+                hb[4 * k + i] = pack2(o2.x - h2.x, o2.y - h2.y);
+              }
+            }
+          }
+          if (c + 32 < c_lo + BN / 2 && n0 + 32 < N) fetch(n0 + 32);
+          // block(s) for this chunk: out alternates between the two when
+          // there is no history stream, else out -> block 0, hist -> block 1
+          uint8_t* b0 = ep + (e.hist_out ? 0 : (epi_cnt & 1) * 2048);
+          if (lane == 0) {
+            if (e.hist_out) bulk_wait_read<0>(); else bulk_wait_read<1>();
+          }
+          __syncwarp();
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            *reinterpret_cast<uint4*>(b0 + blk_off(lane, k)) = make_uint4(ob[4 * k], ob[4 * k + 1], ob[4 * k + 2], ob[4 * k + 3]);
+            if (e.hist_out)
+              *reinterpret_cast<uint4*>(ep + 2048 + blk_off(lane, k)) =
+                  make_uint4(hb[4 * k], hb[4 * k + 1], hb[4 * k + 2], hb[4 * k + 3]);
+          }
+          fence_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store(&tmO, b0, n0, t.m0 + q * 32);
+            if (e.hist_out) tma_store(&tmH, ep + 2048, n0, t.m0 + q * 32);
+            bulk_commit();
+          }
+          ++epi_cnt;
+        }
       } else if constexpr (C::XPOSE_BYTES > 0) {
         // lane = output column n + lane; TMEM column = output row.  Blocks of
         // 16 rows x 32 columns go through the warp's buffer (XOR-swizzled,
         // conflict-free both ways); afterwards lane l holds row l / 2,
         // columns 16 (l % 2) .. + 15.
         const int n = t.n0 + q * 32;
+        if (lane == 0) bulk_wait_read<0>();  // TMA stores of earlier tiles done reading the buffer
+        __syncwarp();
         for (int c = h * (BN / 2); c < (h + 1) * (BN / 2) && n < N; c += 16) {
           const int m0 = t.m0 + c;
           if (m0 >= M) break;
@@ -246,6 +370,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
     }
+    if (C::XPOSE_BYTES > 0 && lane == 0) bulk_wait_all();  // TMA stores complete before exit
   }
   tc_fence_before();
   __syncthreads();
@@ -344,6 +469,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA use
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // dependents may launch once every CTA holds its TMEM; the previous
+  // kernel's outputs are complete after the wait
+  pdl_trigger();
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -473,6 +602,19 @@ bool make_map(CUtensorMap* m, const void* base, int rows, int cols, int ld, int 
   return r == CUDA_SUCCESS;
 }
 
+// Store map of the staged epilogue: [rows, cols] bf16 with row stride ld
+// elements, box 32 x 32, 64-byte swizzle (one block row = 64 bytes).
+bool make_store_map(CUtensorMap* m, void* base, int rows, int cols, int ld) {
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 // Tile width choice: the fewest waves of rows_per_tile x BN tiles over the
 // available CTAs (or CTA pairs), ties to the wider tile (less shared-memory
 // traffic per FLOP).
@@ -506,9 +648,9 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
     const long long tiles = (long long)((M + 2 * BM - 1) / (2 * BM)) * ((N + bn - 1) / bn);
     const int grid = 2 * (int)(tiles < pairs ? tiles : pairs);
     if (bn == 256)
-      k_gemm_tc2<256><<<grid, THREADS, Cfg2<256>::SMEM, s>>>(ma, mb, M, N, K, e);
+      launch_pdl(k_gemm_tc2<256>, grid, THREADS, Cfg2<256>::SMEM, s, ma, mb, M, N, K, e);
     else
-      k_gemm_tc2<128><<<grid, THREADS, Cfg2<128>::SMEM, s>>>(ma, mb, M, N, K, e);
+      launch_pdl(k_gemm_tc2<128>, grid, THREADS, Cfg2<128>::SMEM, s, ma, mb, M, N, K, e);
     return launched();
   }
   // Every tile (128 x 256 full rate, 128 x 128 at half rate, swapped 128 x
@@ -521,7 +663,8 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
   const long long t256 = (long long)tm.num_m * (N / 256) + (rem ? (long long)((rem + 127) / 128) * tm.num_m2 : 0);
   const long long t128 = (long long)tm.num_m * ((N + 127) / 128);
   const bool wide = (t256 + g_sms - 1) / g_sms <= (t128 + g_sms - 1) / g_sms;
-  CUtensorMap mw128 = {}, ma256 = {};
+  CUtensorMap mw128 = {}, ma256 = {}, mo = {}, mh = {};
+  tm.staged = 0;
   if (wide) {
     tm.n_full = N / 256;
     tm.n_norm = tm.num_m * tm.n_full;
@@ -529,15 +672,24 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
     if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, 256)) return cudaErrorInvalidValue;
     if (rem && (!make_map(&mw128, W, N, K, ldw, BM) || !make_map(&ma256, A, M, K, lda, 256)))
       return cudaErrorInvalidValue;
+    // staged (TMA-store) epilogue: one bf16 output of 16-byte aligned rows,
+    // plus the history stream when present
+    const bool aligned = !((uintptr_t)e.out & 15) && e.ldo % 8 == 0 &&
+                         (!e.hist_out || (!((uintptr_t)e.hist_out & 15) && !((uintptr_t)e.hist_base & 15)));
+    // (a warp's 32 rows must span at most two gate rows)
+    const bool gate_ok = !e.gate || ((e.seg_split <= 0 || e.rpb0 >= 32) && e.rpb1 >= 32);
+    if (!e.out_f32 && e.split_col >= N && aligned && gate_ok && make_store_map(&mo, e.out, M, N, e.ldo) &&
+        (!e.hist_out || make_store_map(&mh, e.hist_out, M, N, e.ldo)))
+      tm.staged = 1;
     const int grid = (int)(t256 < g_sms ? t256 : g_sms);
-    k_gemm_tc<256><<<grid, THREADS, Cfg<256>::SMEM, s>>>(ma, mb, mw128, ma256, M, N, K, tm, e);
+    launch_pdl(k_gemm_tc<256>, grid, THREADS, Cfg<256>::SMEM, s, ma, mb, mw128, ma256, mo, mh, M, N, K, tm, e);
   } else {
     tm.n_full = (N + 127) / 128;
     tm.n_norm = tm.num_m * tm.n_full;
     tm.n_tiles = tm.n_norm;
     if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, 128)) return cudaErrorInvalidValue;
     const int grid = (int)(t128 < g_sms ? t128 : g_sms);
-    k_gemm_tc<128><<<grid, THREADS, Cfg<128>::SMEM, s>>>(ma, mb, ma, mb, M, N, K, tm, e);
+    launch_pdl(k_gemm_tc<128>, grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, M, N, K, tm, e);
   }
   return launched();
 }

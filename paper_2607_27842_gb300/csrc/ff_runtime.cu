@@ -93,6 +93,9 @@ struct featfix_ctx {
   std::vector<unsigned char> kinds;
   std::vector<int> keff;
   std::vector<double> wts;
+  std::vector<int> keff_bl;         // per (step, block): FEATFIX_FLAG_SITE_UPDATES_HISTORY
+  std::vector<double> wts_bl;
+  std::vector<int> bhead;           // per block: ring slot of its newest increment
   std::vector<char> isref;
 
   // trajectory state
@@ -219,10 +222,15 @@ void draft_weights(const std::vector<int>& s, int t, bool recursive, double* w) 
   }
 }
 
+// Per step: kinds[i*L + l], the draft order / weights of the refresh-only
+// history (keff[i], wts[i*4 + j]) and, per (step, block), those of the
+// history a draft of that block actually reads (keff_bl[i*L + l],
+// wts_bl[(i*L + l)*4 + j]): the same unless FEATFIX_FLAG_SITE_UPDATES_HISTORY
+// lets a site push its block's increment.
 featfix_status plan_core(int steps, int L, const int* refresh, int n_refresh, int K, const featfix_site* sites,
                          int n_sites, int mode, unsigned flags, std::vector<unsigned char>& kinds,
                          std::vector<int>& keff, std::vector<double>& wts, std::vector<char>& isref,
-                         std::string& err) {
+                         std::vector<int>& keff_bl, std::vector<double>& wts_bl, std::string& err) {
   if (mode < FEATFIX_MODE_FEATFIX || mode > FEATFIX_MODE_VANILLA) { err = "unknown mode"; return FEATFIX_ERR_INVALID_ARG; }
   if (steps < 1 || L < 1) { err = "steps and layers must be positive"; return FEATFIX_ERR_SCHEDULE; }
   if (K < 0 || K > 3) { err = "draft order must be in [0, 3]"; return FEATFIX_ERR_SCHEDULE; }
@@ -247,11 +255,20 @@ featfix_status plan_core(int steps, int L, const int* refresh, int n_refresh, in
   kinds.assign((size_t)steps * L, FEATFIX_PLAN_DRAFT);
   keff.assign(steps, -1);
   wts.assign((size_t)steps * 4, 0.0);
-  std::vector<int> nodes;  // refresh steps, newest first
+  keff_bl.assign((size_t)steps * L, -1);
+  wts_bl.assign((size_t)steps * L * 4, 0.0);
+  const bool recursive = (flags & FEATFIX_FLAG_TAYLOR_RECURSIVE) != 0;
+  const bool site_push = (flags & FEATFIX_FLAG_SITE_UPDATES_HISTORY) != 0 && mode != FEATFIX_MODE_VANILLA;
+  auto push = [K](std::vector<int>& nd, int i) {
+    nd.insert(nd.begin(), i);
+    if ((int)nd.size() > K + 1) nd.resize(K + 1);
+  };
+  std::vector<int> nodes;                // refresh steps, newest first
+  std::vector<std::vector<int>> bnodes(L);  // per block: refreshes (+ its sites)
   for (int i = 0; i < steps; ++i) {
     if (isref[i]) {
-      nodes.insert(nodes.begin(), i);
-      if ((int)nodes.size() > K + 1) nodes.resize(K + 1);
+      push(nodes, i);
+      for (int l = 0; l < L; ++l) push(bnodes[l], i);
     }
     const bool all_exact = mode == FEATFIX_MODE_VANILLA || isref[i];
     for (int l = 0; l < L; ++l) {
@@ -264,7 +281,16 @@ featfix_status plan_core(int steps, int L, const int* refresh, int n_refresh, in
       const int ke = std::min(K, (int)nodes.size() - 1);
       keff[i] = ke;
       std::vector<int> s(nodes.begin(), nodes.begin() + ke + 1);
-      draft_weights(s, i, (flags & FEATFIX_FLAG_TAYLOR_RECURSIVE) != 0, &wts[(size_t)i * 4]);
+      draft_weights(s, i, recursive, &wts[(size_t)i * 4]);
+      for (int l = 0; l < L; ++l) {
+        const std::vector<int>& nd = bnodes[l];
+        const int kb = std::min(K, (int)nd.size() - 1);
+        keff_bl[(size_t)i * L + l] = kb;
+        std::vector<int> sb(nd.begin(), nd.begin() + kb + 1);
+        draft_weights(sb, i, recursive, &wts_bl[((size_t)i * L + l) * 4]);
+        // a site's own draft reads the history before its push
+        if (site_push && kinds[(size_t)i * L + l] == FEATFIX_PLAN_SITE) push(bnodes[l], i);
+      }
     }
   }
   return FEATFIX_OK;
@@ -635,7 +661,8 @@ void* ring_slot(featfix_ctx* c, int l, int slot) {
 
 Hist4 hist_ptrs(featfix_ctx* c, int l, int nt) {
   Hist4 h = {{nullptr, nullptr, nullptr, nullptr}};
-  for (int j = 0; j < nt; ++j) h.p[j] = ring_slot(c, l, ((c->head - j) % c->S + c->S) % c->S);
+  const int hd = c->bhead[l];
+  for (int j = 0; j < nt; ++j) h.p[j] = ring_slot(c, l, ((hd - j) % c->S + c->S) % c->S);
   return h;
 }
 
@@ -680,6 +707,7 @@ featfix_status verify_shadow(featfix_ctx* ctx, int i, int nt, const float* wf) {
 featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* cond) {
   if (i == 0) {
     ctx->head = ctx->S - 1;
+    ctx->bhead.assign(ctx->L, ctx->S - 1);
     ctx->count = 0;
     ctx->cnt = {0, 0, 0, 0};
     ctx->log_sites.clear();
@@ -690,14 +718,21 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
   const size_t bytes = (size_t)ctx->E * ctx->es;
   FF_TRY(embed(ctx, latent, cond, ctx->x0buf));
   const int new_slot = (ctx->head + 1) % ctx->S;
-  const int nt = ctx->keff[i] + 1;
+  const bool site_push = (ctx->flags & FEATFIX_FLAG_SITE_UPDATES_HISTORY) != 0;
+  int nt = ctx->keff[i] + 1;
   float wf[4];
   for (int j = 0; j < 4; ++j) wf[j] = (float)ctx->wts[(size_t)i * 4 + j];
+  // block l's draft order and weights (its own history when sites push)
+  auto block_weights = [&](int l) {
+    if (!site_push) return;
+    nt = ctx->keff_bl[(size_t)i * L + l] + 1;
+    for (int j = 0; j < 4; ++j) wf[j] = (float)ctx->wts_bl[((size_t)i * L + l) * 4 + j];
+  };
   bool has_site = false, has_capture = false;
   for (int l = 0; l < L; ++l) has_site |= ctx->kinds[(size_t)i * L + l] == FEATFIX_PLAN_SITE;
   for (auto& cp : ctx->caps) has_capture |= cp.step == i;
-  const bool telescope = !refresh && !vanilla && !has_capture && !(ctx->flags & FEATFIX_FLAG_PER_BLOCK_DRAFT) &&
-                         (!has_site || ctx->mode == FEATFIX_MODE_VERIFY);
+  const bool telescope = !refresh && !vanilla && !has_capture && !site_push &&
+                         !(ctx->flags & FEATFIX_FLAG_PER_BLOCK_DRAFT) && (!has_site || ctx->mode == FEATFIX_MODE_VERIFY);
   void* x = ctx->x0buf;
   if (telescope) {
     if (has_site) FF_TRY(verify_shadow(ctx, i, nt, wf));
@@ -715,15 +750,20 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
       for (auto& cp : ctx->caps)
         if (cp.step == i && cp.layer == l && cp.in) FF_CK(cudaMemcpyAsync(cp.in, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
       const unsigned char kind = ctx->kinds[(size_t)i * L + l];
+      const int bslot = (ctx->bhead[l] + 1) % ctx->S;  // block l's next ring slot
       if (kind == FEATFIX_PLAN_EXACT) {
-        void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, new_slot) : nullptr;
+        void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, bslot) : nullptr;
         FF_TRY(exact_block(ctx, i, l, x, y, hist));
         advance();
       } else if (kind == FEATFIX_PLAN_DRAFT) {
+        block_weights(l);
         KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
         FF_CK(launch_draft(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
       } else {
-        FF_TRY(exact_block(ctx, i, l, x, y, nullptr));
+        block_weights(l);
+        // with site pushes the exact increment goes to the spare slot; the
+        // draft below still reads the K_eff + 1 entries before it
+        FF_TRY(exact_block(ctx, i, l, x, y, site_push ? ring_slot(ctx, l, bslot) : nullptr));
         ctx->cnt.paid_checks++;
         if (ctx->mode != FEATFIX_MODE_EXACT_ONLY) {
           const int slot = (int)ctx->log_sites.size();
@@ -738,6 +778,7 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
           advance();
           ctx->cnt.forwarded++;
         }
+        if (site_push) ctx->bhead[l] = bslot;
       }
       for (auto& cp : ctx->caps)
         if (cp.step == i && cp.layer == l && cp.out) FF_CK(cudaMemcpyAsync(cp.out, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
@@ -747,6 +788,7 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
     KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
     FF_CK(launch_diff(ctx->dt, x, ctx->x0buf, off(ctx->sring, (long long)new_slot * ctx->E, ctx->es), ctx->E, ctx->st));
     ctx->head = new_slot;
+    for (int l = 0; l < L; ++l) ctx->bhead[l] = (ctx->bhead[l] + 1) % ctx->S;
     ctx->count = std::min(ctx->count + 1, ctx->S);
   }
   if (refresh || vanilla) ctx->cnt.refresh_steps++;
@@ -929,9 +971,11 @@ featfix_status create_impl(featfix_ctx* ctx) {
 }
 
 // Per-schedule device state: history ring, modulation tables, logs.
-featfix_status schedule_buffers(featfix_ctx* ctx, int steps, int K, int mode, int n_sites) {
+featfix_status schedule_buffers(featfix_ctx* ctx, int steps, int K, int mode, int n_sites, unsigned flags) {
   const int es = ctx->es, C = ctx->C, Bm = ctx->Bm;
-  const int S = K + 1;
+  // K + 1 increments per block; a site that pushes its increment writes a
+  // slot while its own draft still reads the K + 1 newest: one spare slot
+  const int S = K + 1 + ((flags & FEATFIX_FLAG_SITE_UPDATES_HISTORY) ? 1 : 0);
   if (ctx->ring && ctx->S != S) {
     free_ptr(&ctx->ring);
     free_ptr(&ctx->sring);
@@ -1011,16 +1055,32 @@ featfix_status featfix_plan_build(int steps, int n_layers_, const int* refresh, 
                                   const featfix_site* sites, int n_sites, int mode, unsigned flags,
                                   unsigned char* kinds, int* k_eff, double* weights) {
   std::vector<unsigned char> kd;
-  std::vector<int> ke;
-  std::vector<double> wt;
+  std::vector<int> ke, keb;
+  std::vector<double> wt, wtb;
   std::vector<char> isref;
   std::string err;
   featfix_status s = plan_core(steps, n_layers_, refresh, n_refresh, draft_order, sites, n_sites, mode, flags, kd, ke,
-                               wt, isref, err);
+                               wt, isref, keb, wtb, err);
   if (s != FEATFIX_OK) return s;
   if (kinds) std::memcpy(kinds, kd.data(), kd.size());
   if (k_eff) std::memcpy(k_eff, ke.data(), ke.size() * sizeof(int));
   if (weights) std::memcpy(weights, wt.data(), wt.size() * sizeof(double));
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_plan_build_blocks(int steps, int n_layers_, const int* refresh, int n_refresh, int draft_order,
+                                         const featfix_site* sites, int n_sites, int mode, unsigned flags, int* k_eff,
+                                         double* weights) {
+  std::vector<unsigned char> kd;
+  std::vector<int> ke, keb;
+  std::vector<double> wt, wtb;
+  std::vector<char> isref;
+  std::string err;
+  featfix_status s = plan_core(steps, n_layers_, refresh, n_refresh, draft_order, sites, n_sites, mode, flags, kd, ke,
+                               wt, isref, keb, wtb, err);
+  if (s != FEATFIX_OK) return s;
+  if (k_eff) std::memcpy(k_eff, keb.data(), keb.size() * sizeof(int));
+  if (weights) std::memcpy(weights, wtb.data(), wtb.size() * sizeof(double));
   return FEATFIX_OK;
 }
 
@@ -1080,12 +1140,12 @@ featfix_status featfix_set_schedule(featfix_ctx* ctx, int steps, const int* refr
                                     const featfix_site* sites, int n_sites, int mode, unsigned flags) {
   if (!ctx) return FEATFIX_ERR_INVALID_ARG;
   std::vector<unsigned char> kd;
-  std::vector<int> ke;
-  std::vector<double> wt;
+  std::vector<int> ke, keb;
+  std::vector<double> wt, wtb;
   std::vector<char> isref;
   std::string err;
   featfix_status s = plan_core(steps, ctx->L, refresh, n_refresh, draft_order, sites, n_sites, mode, flags, kd, ke, wt,
-                               isref, err);
+                               isref, keb, wtb, err);
   if (s != FEATFIX_OK) return fail(ctx, s, err);
   if (ctx->d.sampler == FEATFIX_SAMPLER_DDIM && (1000 % steps != 0))
     return fail(ctx, FEATFIX_ERR_UNSUPPORTED, "DDIM needs steps dividing 1000");
@@ -1101,7 +1161,7 @@ featfix_status featfix_set_schedule(featfix_ctx* ctx, int steps, const int* refr
     if (any) need[i] = nn++;
   }
   ctx->n_need = nn;
-  FF_TRY(schedule_buffers(ctx, steps, draft_order, mode, n_sites));
+  FF_TRY(schedule_buffers(ctx, steps, draft_order, mode, n_sites, flags));
   ctx->need_row = need;
   ctx->steps = steps;
   std::vector<float> times(steps);
@@ -1111,6 +1171,8 @@ featfix_status featfix_set_schedule(featfix_ctx* ctx, int steps, const int* refr
   ctx->kinds.swap(kd);
   ctx->keff.swap(ke);
   ctx->wts.swap(wt);
+  ctx->keff_bl.swap(keb);
+  ctx->wts_bl.swap(wtb);
   ctx->isref.swap(isref);
   ctx->K = draft_order;
   ctx->mode = mode;

@@ -39,13 +39,27 @@ __device__ __forceinline__ bool mbar_try(uint64_t* b, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait on phase `parity`; false (and the CTA abort flag raised) on
-// timeout or when another role already aborted.
+// Non-blocking probe of phase `parity`: never suspends the thread, for
+// hand-offs where the wake-up latency of a suspended try_wait would sit on
+// the critical path.
+__device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(saddr(b)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait on phase `parity` (SPIN: poll with test_wait instead of a
+// suspending try_wait); false (and the CTA abort flag raised) on timeout or
+// when another role already aborted.
+template <bool SPIN = false>
 static __device__ __noinline__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, unsigned int* watchdog) {
-  if (mbar_try(b, parity)) return true;
+  if (SPIN ? mbar_test(b, parity) : mbar_try(b, parity)) return true;
   const unsigned long long t0 = gtimer();
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try(b, parity)) return true;
+    if (SPIN ? mbar_test(b, parity) : mbar_try(b, parity)) return true;
     if ((it & 63) == 0) {
       if (*abort_flag) return false;
       if (gtimer() - t0 > WAIT_LIMIT_NS) {
@@ -66,6 +80,23 @@ __device__ __forceinline__ void tma_load(const CUtensorMap* tm, uint64_t* bar, v
 }
 
 // ---- CTA-pair (2-SM) helpers --------------------------------------------------
+// TMA tile store shared -> global (bulk async-group of the issuing thread);
+// rows / columns outside the tensor are not written
+__device__ __forceinline__ void tma_store(const CUtensorMap* tm, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"((uint64_t)tm),
+               "r"(x), "r"(y), "r"(saddr(src))
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// wait until at most N of this thread's bulk groups still read shared memory
+template <int N> __device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// wait until all of this thread's bulk groups completed (writes visible)
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// generic-proxy shared-memory writes -> visible to the async proxy (TMA)
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));

@@ -22,6 +22,7 @@ SAMPLER = {"euler": 0, "ddim": 1}
 PLAN_EXACT, PLAN_DRAFT, PLAN_SITE = 0, 1, 2
 FLAG_TAYLOR_RECURSIVE = 1
 FLAG_PER_BLOCK_DRAFT = 2
+FLAG_SITE_UPDATES_HISTORY = 4
 KCLASS = {"gemm": 0, "attention": 1, "draft": 2, "verify": 3, "other": 4}
 
 
@@ -71,6 +72,7 @@ SIGNATURES = {
     "featfix_get_plan": (_I, [_VP, _P(ctypes.c_ubyte), _P(_I), _P(_D)]),
     "featfix_plan_build": (_I, [_I, _I, _P(_I), _I, _I, _P(Site), _I, _I, ctypes.c_uint, _P(ctypes.c_ubyte),
                                 _P(_I), _P(_D)]),
+    "featfix_plan_build_blocks": (_I, [_I, _I, _P(_I), _I, _I, _P(Site), _I, _I, ctypes.c_uint, _P(_I), _P(_D)]),
     "featfix_debug_capture": (_I, [_VP, _I, _I, _VP, _VP]),
     "featfix_debug_block": (_I, [_VP, _I, _I, _VP, _VP, _VP]),
     "featfix_token_row": (_LL, [_P(ModelDesc), _I, _I]),
@@ -267,6 +269,19 @@ def featfix_get_plan(ctx, steps, n_layers):
     return kinds.reshape(steps, n_layers), keff, w.reshape(steps, 4)
 
 
+def featfix_plan_build_blocks(steps, n_layers, refresh, draft_order, sites, mode="featfix", flags=0):
+    """Host-only per-block draft plan: (k_eff [steps, L], weights [steps, L, 4])."""
+    import numpy as np
+    ref = (_I * max(len(refresh), 1))(*[int(r) for r in refresh])
+    sa, ns = _sites_arr(sites)
+    keff = np.zeros(steps * n_layers, dtype=np.int32)
+    w = np.zeros(steps * n_layers * 4, dtype=np.float64)
+    m = MODES[mode] if isinstance(mode, str) else int(mode)
+    _check(lib().featfix_plan_build_blocks(int(steps), int(n_layers), ref, len(refresh), int(draft_order), sa, ns, m,
+                                           int(flags), keff.ctypes.data_as(_P(_I)), w.ctypes.data_as(_P(_D))))
+    return keff.reshape(steps, n_layers), w.reshape(steps, n_layers, 4)
+
+
 def featfix_plan_build(steps, n_layers, refresh, draft_order, sites, mode="featfix", flags=0):
     """Host-only plan: (kinds [steps, L] uint8, k_eff [steps], weights [steps, 4])."""
     import numpy as np
@@ -280,6 +295,19 @@ def featfix_plan_build(steps, n_layers, refresh, draft_order, sites, mode="featf
                                     int(flags), kinds.ctypes.data_as(_P(ctypes.c_ubyte)),
                                     keff.ctypes.data_as(_P(_I)), w.ctypes.data_as(_P(_D))))
     return kinds.reshape(steps, n_layers), keff, w.reshape(steps, 4)
+
+
+def featfix_plan_build_blocks(steps, n_layers, refresh, draft_order, sites, mode="featfix", flags=0):
+    """Host-only per-block draft plan: (k_eff [steps, L], weights [steps, L, 4])."""
+    import numpy as np
+    ref = (_I * max(len(refresh), 1))(*[int(r) for r in refresh])
+    sa, ns = _sites_arr(sites)
+    keff = np.zeros(steps * n_layers, dtype=np.int32)
+    w = np.zeros(steps * n_layers * 4, dtype=np.float64)
+    m = MODES[mode] if isinstance(mode, str) else int(mode)
+    _check(lib().featfix_plan_build_blocks(int(steps), int(n_layers), ref, len(refresh), int(draft_order), sa, ns, m,
+                                           int(flags), keff.ctypes.data_as(_P(_I)), w.ctypes.data_as(_P(_D))))
+    return keff.reshape(steps, n_layers), w.reshape(steps, n_layers, 4)
 
 
 def featfix_debug_capture(ctx, step, layer, dev_in, dev_out):

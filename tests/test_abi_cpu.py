@@ -128,6 +128,38 @@ def test_recursive_flag_matches_oracle_variant(lib):
         np.testing.assert_allclose(w[i, :len(ref)], ref, rtol=1e-12, atol=1e-12)
 
 
+@pytest.mark.parametrize("name", list(syn.SHAPES))
+@pytest.mark.parametrize("mode", ["featfix", "verify", "exact_only"])
+@pytest.mark.parametrize("push", [False, True])
+def test_block_plan_matches_oracle_histories(lib, name, mode, push):
+    """Per-(step, block) draft weights against the oracle's per-block history
+    steps, with and without sites pushing their increments."""
+    wl = syn.workload(name)
+    L = wl.shape.n_layers
+    flags = ff.FLAG_SITE_UPDATES_HISTORY if push else 0
+    keff, w = ff.featfix_plan_build_blocks(wl.steps, L, wl.refresh, wl.K, wl.sites, mode, flags)
+    _, keff_step, w_step = ff.featfix_plan_build(wl.steps, L, wl.refresh, wl.K, wl.sites, mode, flags)
+    hs = osched.block_history_steps(wl.steps, L, wl.refresh, wl.K, wl.sites, mode, push)
+    site_set = {tuple(x) for x in wl.sites}
+    for i in range(wl.steps):
+        for l in range(L):
+            if hs[i][l] is None:
+                assert keff[i, l] == -1
+                continue
+            assert keff[i, l] == len(hs[i][l]) - 1 == min(wl.K, len(hs[i][l]) - 1)
+            ref = implied_weights(i, hs[i][l], "interp")
+            np.testing.assert_allclose(w[i, l, :len(ref)], ref, rtol=1e-12, atol=1e-12)
+            if not push:   # without pushes every block reads the refresh-only history
+                assert keff[i, l] == keff_step[i]
+                np.testing.assert_array_equal(w[i, l], w_step[i])
+    if push and wl.sites:
+        # a block whose site precedes a drafted step reads that site step
+        i0, l0 = sorted(site_set)[0]
+        later = [i for i in range(i0 + 1, wl.steps) if i not in wl.refresh]
+        if later and later[0] < min([r for r in wl.refresh if r > i0], default=wl.steps):
+            assert hs[later[0]][l0][0] == i0
+
+
 @pytest.mark.parametrize("bad,status", [
     (dict(refresh=(1, 3)), ff.ERR_SCHEDULE),
     (dict(sites=((3, 0),)), ff.ERR_SCHEDULE),

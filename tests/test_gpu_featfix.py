@@ -77,6 +77,27 @@ def test_sample_matches_oracle(case):
         assert log_close(g["rel_l2"], r["rel_l2"], case.sh.dtype), (g, r)
 
 
+@pytest.mark.parametrize("mode", ["featfix", "verify"])
+def test_site_history_push_matches_oracle(case, mode):
+    """FEATFIX_FLAG_SITE_UPDATES_HISTORY: sites push their exact increment
+    onto their block's history; trajectory, logs and accounting against the
+    oracle run with the same reading."""
+    flags = ff.FLAG_SITE_UPDATES_HISTORY
+    case.schedule(mode, flags=flags)
+    lat = case.sample(seed=1)
+    logs, cnt = ff.featfix_get_log(case.ctx)
+    x_ref, logs_ref, cnt_ref = case.oracle_run(mode, seed=1, site_updates_history=True)
+    err = rel_l2(lat.cpu().numpy(), x_ref)
+    assert err < tol_latent(case.sh), err
+    assert {k: cnt[k] for k in cnt_ref} == cnt_ref
+    assert [(e["step"], e["layer"]) for e in logs] == [(e["step"], e["layer"]) for e in logs_ref]
+    for g, r in zip(logs, logs_ref):
+        assert log_close(g["rel_l1"], r["rel_l1"], case.sh.dtype), (g, r)
+    # the reading changes the trajectory when a site precedes a drafted step
+    x_def, _, _ = case.oracle_run(mode, seed=1)
+    assert np.abs(x_ref - x_def).max() > 0
+
+
 def test_blocks_teacher_forced(case):
     """Every block of the trajectory on the GPU's own incoming state: exact
     blocks vs B_l (Eq. 1), drafts vs Eq. 2 over the GPU's refresh increments."""

@@ -209,6 +209,11 @@ ATTN_CASES = [
     ("bf16", 2, 77, 1000, 2, 128),
     ("bf16", 1, 0, 1100, 3, 72),
     ("bf16", 2, 130, 1030, 2, 64),
+    # full-size attention of two workloads: DiT-XL/2 (256 image tokens, 16
+    # heads x 72, model batch 16) and FLUX (512 text + 4096 image tokens,
+    # 24 heads x 128)
+    ("bf16", 16, 0, 256, 16, 72),
+    ("bf16", 1, 512, 4096, 24, 128),
 ]
 
 
@@ -227,7 +232,11 @@ def test_attention_matches_oracle(cuda, dtype, B, nt, ni, H, d):
     q = Q[..., :C].reshape(B, nt + ni, H, d).transpose(0, 2, 1, 3)
     k = Q[..., C:2 * C].reshape(B, nt + ni, H, d).transpose(0, 2, 1, 3)
     v = Q[..., 2 * C:3 * C].reshape(B, nt + ni, H, d).transpose(0, 2, 1, 3)
-    ref = oracle.model.merge_heads(oracle.model.attention(q, k, v))
-    got = f64(out)[rows][..., :C]
-    assert rel_l2(got, ref) < (1e-5 if dtype == "f32" else 1e-2)
+    got = f64(out)[rows][..., :C].reshape(B, nt + ni, H, d)
+    # long sequences: the float64 score matrix of every head would not fit,
+    # so the first, a middle and the last head are checked
+    heads = range(H) if B * H * (nt + ni) ** 2 <= 5e7 else sorted({0, H // 2, H - 1})
+    for h in heads:
+        ref = oracle.model.attention(q[:, h:h + 1], k[:, h:h + 1], v[:, h:h + 1])[:, 0]
+        assert rel_l2(got[:, :, h], ref) < (1e-5 if dtype == "f32" else 1e-2), h
     assert np.all(f64(out)[:, C:] == 0)        # nothing written past C

@@ -527,6 +527,35 @@ def test_featfix_and_verify_agree_until_the_first_site_then_differ():
     assert np.abs(a - b).max() > 0
 
 
+def test_site_history_push_reading():
+    """SITE_UPDATES_HISTORY reading: with reuse (K = 0) a block's next draft
+    after its site adds exactly the site's exact increment h_f - u; by
+    default it adds the last refresh increment.  A site's own draft and
+    logged discrepancy do not depend on the reading."""
+    wl, sh, W, cond, xT = tiny_setup()
+    (i0, l0) = sorted(wl.sites)[0]
+    nxt = i0 + 1
+    assert nxt not in wl.refresh
+    for push in (False, True):
+        inc = {}
+        def hook(i, l, kind, u, h, extra):
+            if l == l0 and kind != schedule.DRAFT or (l == l0 and i == nxt):
+                inc[(i, kind)] = ((extra["h_f"] if extra else h) - u, h - u)
+        _, logs, _ = featfix.run(W, sh, cond, xT, wl.steps, wl.refresh, 0, wl.sites, "verify", hook=hook,
+                                 site_updates_history=push)
+        draft_inc = inc[(nxt, schedule.DRAFT)][1]
+        site_exact = inc[(i0, schedule.SITE)][0]
+        last_ref = max(r for r in wl.refresh if r < i0)
+        refresh_inc = inc[(last_ref, schedule.EXACT)][0]
+        # (h - u recovers the added increment up to the rounding of u + R)
+        want = site_exact if push else refresh_inc
+        np.testing.assert_allclose(draft_inc, want, rtol=0, atol=1e-15)
+        assert np.abs(site_exact - refresh_inc).max() > 0
+        if not push:
+            base = logs
+    assert logs[0]["rel_l1"] == base[0]["rel_l1"]
+
+
 def test_discrepancy_definitions():
     hf = np.array([1.0, -2.0, 3.0])
     hd = np.array([1.5, -2.0, 2.0])
