@@ -47,6 +47,9 @@ def parse():
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--mode", default="featfix", choices=["featfix", "verify", "exact_only", "vanilla"])
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--sweep", choices=["resolution"], default=None,
+                   help="instead of the headline line: one line per FLUX resolution (512^2, 768^2, 1024^2) with "
+                        "sampling rate and device memory")
     return p.parse_args()
 
 
@@ -268,8 +271,55 @@ def profile_traffic():
     return tr if hsh == digest else None
 
 
+def run_sweep(args):
+    """Latency and device memory of the FLUX-shaped cached sampler over image
+    resolutions (the paper's resolution study): per resolution one JSON line
+    with denoise steps/s, ms per sampling run, the bf16 weights, the
+    library's own device memory (history ring, activations, workspaces) and
+    the total device memory the run holds."""
+    import torch
+    from paper_2607_27842_gb300 import featfix as ff, synthetic as syn
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    for name, img in (("flux_512", 512), ("flux_768", 768), ("flux", 1024)):
+        wl = syn.workload(name)
+        sh = wl.shape
+        torch.cuda.synchronize(dev)
+        torch.cuda.empty_cache()
+        free0 = torch.cuda.mem_get_info(dev)[0]
+        weights = syn.make_weights(sh, seed=0, device=dev)
+        cond = syn.make_cond(sh, seed=2, device=dev)
+        lat = torch.empty(sh.latent_dims, dtype=torch.float32, device=dev)
+        torch.cuda.synchronize(dev)
+        free1 = torch.cuda.mem_get_info(dev)[0]
+        ctx = ff.featfix_create(sh, weights, stream)
+        ff.featfix_set_schedule(ctx, wl.steps, wl.refresh, wl.K, wl.sites, args.mode)
+        for i in range(max(1, args.warmup)):
+            ff.featfix_sample(ctx, 1000 + i, wl.steps, cond, lat)
+        torch.cuda.synchronize(dev)
+        free2 = torch.cuda.mem_get_info(dev)[0]
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for i in range(args.steps):
+            ff.featfix_sample(ctx, 1 + i, wl.steps, cond, lat)
+        ev1.record(stream)
+        torch.cuda.synchronize(dev)
+        ms = ev0.elapsed_time(ev1) / args.steps
+        wbytes = sum(t.numel() * t.element_size() for t in weights.values())
+        print(json.dumps({"sweep": "resolution", "workload": name, "image": "%dx%d" % (img, img),
+                          "tokens": sh.tokens, "mode": args.mode, "value": wl.steps / (ms / 1e3), "unit": UNIT,
+                          "ms_per_sample": ms, "weights_gb": wbytes / 1e9, "library_gb": (free1 - free2) / 1e9,
+                          "device_gb": (free0 - free2) / 1e9, "steps": args.steps}), flush=True)
+        ff.featfix_destroy(ctx)
+        del weights, cond, lat
+
+
 def main():
     args = parse()
+    if args.sweep:
+        run_sweep(args)
+        return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))

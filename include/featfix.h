@@ -257,6 +257,25 @@ FEATFIX_API featfix_status featfix_plan_build(int steps, int n_layers, const int
                                   int mode, unsigned flags, unsigned char* kinds, int* k_eff,
                                   double* weights);
 
+/* Partial forwarding arms (the token- and channel-level alternatives to
+ * whole-block forwarding the paper compares against, Section 3.2): at a
+ * FeatFix site the forwarded output takes the exact block output h^f only
+ * on the selected tokens or channels and the draft h^d elsewhere (the
+ * discrepancy of Eq. 4 is still taken over the whole tensor).  The paper
+ * does not say which tokens or channels are selected, so the caller passes
+ * the selection.
+ *  axis  FEATFIX_MASK_NONE: whole-block forwarding (Eq. 5, the default).
+ *        FEATFIX_MASK_TOKENS: mask[n], n = 0 .. txt_tokens + image tokens - 1
+ *        in a sample's sequence order (text first), the same for every
+ *        sample of the model batch.
+ *        FEATFIX_MASK_CHANNELS: mask[c], c = 0 .. hidden - 1.
+ *  mask  host bytes, nonzero = forward h^f; copied (the call synchronises
+ *        the context stream and drops a captured trajectory graph).
+ * Only the FeatFix arm uses the mask.  Errors: INVALID_ARG for an unknown
+ * axis, a null mask or a length other than the axis' size.                  */
+enum { FEATFIX_MASK_NONE = 0, FEATFIX_MASK_TOKENS = 1, FEATFIX_MASK_CHANNELS = 2 };
+FEATFIX_API featfix_status featfix_set_forward_mask(featfix_ctx* ctx, int axis, const unsigned char* mask, int n);
+
 /* Host-only: per (step, block) draft order k_eff [steps*n_layers] (-1
  * where the block is exact) and weights [steps*n_layers*4] of the history
  * that block's draft reads.  Equal to featfix_plan_build's per-step values

@@ -51,8 +51,19 @@ def model_input(shape, x):
     return np.concatenate([x, x], axis=0) if shape.cfg else x
 
 
+def forward_partial(hd, hf, mask):
+    """Token- or channel-level partial forwarding arm (Section 3.2's
+    alternatives to whole-block forwarding): the exact output on the
+    selected tokens (axis 'tokens', mask over a sample's sequence) or
+    channels (axis 'channels'), the draft elsewhere."""
+    axis, m = mask
+    m = np.asarray(m, dtype=bool)
+    sel = m[None, :, None] if axis == "tokens" else m[None, None, :]
+    return np.where(sel, hf, hd)
+
+
 def run(W, shape, cond, x_T, steps, refresh, K, sites, mode="featfix",
-        variant="interp", hook=None, site_updates_history=False):
+        variant="interp", hook=None, site_updates_history=False, forward_mask=None):
     """Run the cached sampler.
 
     W      dict of float64 weights.
@@ -62,6 +73,8 @@ def run(W, shape, cond, x_T, steps, refresh, K, sites, mode="featfix",
     hook   optional callable(step, layer, kind, u, h_out, extra) for tests.
     site_updates_history   push a site's exact increment onto its block's
            history (after the site's own draft).
+    forward_mask  None (whole-block forwarding) or ('tokens', mask[N_tot]) /
+           ('channels', mask[C]): the FeatFix arm forwards h_f only there.
 
     Returns (x_0, logs, counters) with logs = list of dicts
     {step, layer, rel_l1, rel_l2} in execution order and counters =
@@ -105,7 +118,7 @@ def run(W, shape, cond, x_T, steps, refresh, K, sites, mode="featfix",
                     hd = _draft.draft(u, hist[l], i, K, variant)
                     logs.append({"step": i, "layer": l, "rel_l1": rel_l1(hd, hf), "rel_l2": rel_l2(hd, hf)})
                     if mode == "featfix":
-                        h = hf
+                        h = hf if forward_mask is None else forward_partial(hd, hf, forward_mask)
                         counters["forwarded"] += 1
                     else:
                         h = hd

@@ -267,8 +267,17 @@ inline cudaError_t launched() {
 cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int nt, long long n, cudaStream_t s);
 cudaError_t launch_diff(DType dt, const void* a, const void* b, void* out, long long n, cudaStream_t s);
 size_t verify_workspace_bytes(long long n);
+// Partial forwarding at a site: out <- h_f on selected rows (rmask, per
+// token row) or columns (cmask), h_d elsewhere; row width C.
+struct FwdMix {
+  void* out;
+  const unsigned char* rmask;
+  const unsigned char* cmask;
+  int C;
+};
 cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
-                          int write_draft, double* sums, void* ws, cudaStream_t s);
+                          int write_draft, double* sums, void* ws, cudaStream_t s,
+                          const FwdMix* mix = nullptr);
 cudaError_t launch_ln_mod(DType dt, const void* x, void* out, long long rows, int C, const float* shift,
                           const float* scale, int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s);
 // Sinusoidal features of S model times (device array) -> [S, 256] in dt.

@@ -166,10 +166,15 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// Partial forwarding (token- or channel-level arm): mix != nullptr gets
+// h_f where the element's row (rmask) or column (cmask) is selected and h_d
+// elsewhere; mix may be the h_f buffer itself (each element is read, then
+// written, by the same thread).
 template <class T, int NT>
 __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_THREADS)
-    k_verify(T* __restrict__ u, Hist4 h, float w0, float w1, float w2, float w3, const T* __restrict__ hf,
-             long long n, int write_draft, double* __restrict__ partials) {
+    k_verify(T* __restrict__ u, Hist4 h, float w0, float w1, float w2, float w3, const T* hf,
+             long long n, int write_draft, double* __restrict__ partials, T* mix,
+             const unsigned char* __restrict__ rmask, const unsigned char* __restrict__ cmask, int C) {
   pdl_trigger();
   pdl_wait();
   constexpr int V = VecN<T>::n;
@@ -191,6 +196,15 @@ __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_
       s3 += f[q] * f[q];
     }
     if (write_draft) st16(u + i * V, a);
+    if (mix) {  // C % V == 0: the vector lies in one row
+      const long long e0 = i * V;
+      const long long r = e0 / C;
+      const int c0 = (int)(e0 - r * C);
+      float o[V];
+#pragma unroll
+      for (int q = 0; q < V; ++q) o[q] = (rmask ? rmask[r] : cmask[c0 + q]) ? f[q] : a[q];
+      st16(mix + i * V, o);
+    }
   }
   if (blockIdx.x == 0 && threadIdx.x < n - nvec * V) {
     const long long i = nvec * V + threadIdx.x;
@@ -199,6 +213,7 @@ __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_
     const float d = a - f;
     s0 += fabsf(d); s1 += fabsf(f); s2 += d * d; s3 += f * f;
     if (write_draft) u[i] = from_f<T>(a);
+    if (mix) mix[i] = from_f<T>((rmask ? rmask[i / C] : cmask[i % C]) ? f : a);
   }
   s0 = warp_sum(s0); s1 = warp_sum(s1); s2 = warp_sum(s2); s3 = warp_sum(s3);
   __shared__ float wsum[VERIFY_THREADS / 32][4];
@@ -236,16 +251,21 @@ __global__ void k_verify_finish(const double* __restrict__ partials, int nparts,
 
 template <class T>
 static cudaError_t verify_t(void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
-                           int write_draft, double* sums, void* ws, cudaStream_t s) {
+                           int write_draft, double* sums, void* ws, cudaStream_t s, const FwdMix* fm) {
   const int grid = verify_grid(n);
   double* parts = reinterpret_cast<double*>(ws);
   T* up = reinterpret_cast<T*>(u);
   const T* fp = reinterpret_cast<const T*>(hf);
+  T* mx = fm ? reinterpret_cast<T*>(fm->out) : nullptr;
+  const unsigned char* rm = fm ? fm->rmask : nullptr;
+  const unsigned char* cm = fm ? fm->cmask : nullptr;
+  const int C = fm ? fm->C : 1;
+  if (mx && (C <= 0 || C % VecN<T>::n != 0 || (!rm && !cm) || n % C != 0)) return cudaErrorInvalidValue;
   switch (nt) {
-    case 1: launch_pdl(k_verify<T, 1>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
-    case 2: launch_pdl(k_verify<T, 2>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
-    case 3: launch_pdl(k_verify<T, 3>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
-    case 4: launch_pdl(k_verify<T, 4>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts); break;
+    case 1: launch_pdl(k_verify<T, 1>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C); break;
+    case 2: launch_pdl(k_verify<T, 2>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C); break;
+    case 3: launch_pdl(k_verify<T, 3>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C); break;
+    case 4: launch_pdl(k_verify<T, 4>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C); break;
     default: return cudaErrorInvalidValue;
   }
   cudaError_t e = launched();
@@ -255,10 +275,10 @@ static cudaError_t verify_t(void* u, const Hist4& h, const float* w, int nt, con
 }
 
 cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
-                          int write_draft, double* sums, void* ws, cudaStream_t s) {
+                          int write_draft, double* sums, void* ws, cudaStream_t s, const FwdMix* mix) {
   if (n <= 0) return cudaErrorInvalidValue;
-  return dt == F32 ? verify_t<float>(u, h, w, nt, hf, n, write_draft, sums, ws, s)
-                   : verify_t<bf16>(u, h, w, nt, hf, n, write_draft, sums, ws, s);
+  return dt == F32 ? verify_t<float>(u, h, w, nt, hf, n, write_draft, sums, ws, s, mix)
+                   : verify_t<bf16>(u, h, w, nt, hf, n, write_draft, sums, ws, s, mix);
 }
 
 // ---------------------------------------------------------------------------

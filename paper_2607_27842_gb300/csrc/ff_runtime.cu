@@ -96,6 +96,9 @@ struct featfix_ctx {
   std::vector<int> keff_bl;         // per (step, block): FEATFIX_FLAG_SITE_UPDATES_HISTORY
   std::vector<double> wts_bl;
   std::vector<int> bhead;           // per block: ring slot of its newest increment
+  int fmask_axis = FEATFIX_MASK_NONE;  // partial forwarding at FeatFix sites
+  unsigned char* d_rmask = nullptr;    // [T] per token row (FEATFIX_MASK_TOKENS)
+  unsigned char* d_cmask = nullptr;    // [C] per channel (FEATFIX_MASK_CHANNELS)
   std::vector<char> isref;
 
   // trajectory state
@@ -769,9 +772,13 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
           const int slot = (int)ctx->log_sites.size();
           if (slot >= ctx->max_logs) return fail(ctx, FEATFIX_ERR_STATE, "log overflow");
           const int wr = ctx->mode == FEATFIX_MODE_VERIFY ? 1 : 0;
-          KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 2 + wr) * bytes);
+          // partial forwarding arm: h_f only on the selected tokens / channels
+          const bool partial = ctx->mode == FEATFIX_MODE_FEATFIX && ctx->fmask_axis != FEATFIX_MASK_NONE;
+          const FwdMix fm = {y, ctx->fmask_axis == FEATFIX_MASK_TOKENS ? ctx->d_rmask : nullptr,
+                             ctx->fmask_axis == FEATFIX_MASK_CHANNELS ? ctx->d_cmask : nullptr, ctx->C};
+          KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 2 + wr + (partial ? 1 : 0)) * bytes);
           FF_CK(launch_verify(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, y, ctx->E, wr, ctx->dsums + 4 * slot,
-                              ctx->vws, ctx->st));
+                              ctx->vws, ctx->st, partial ? &fm : nullptr));
           ctx->log_sites.push_back({i, l});
         }
         if (ctx->mode != FEATFIX_MODE_VERIFY) {
@@ -843,7 +850,7 @@ void free_all(featfix_ctx* c) {
   void* bufs[] = {c->xa, c->xb, c->xm, c->qkv, c->att, c->u1, c->big, c->patches, c->pos, c->mout, c->rope,
                   c->ring, c->sring, c->x0buf, c->shadow, c->wmod, c->bmod, c->d_times, c->d_need, c->sin_tab, c->thid_tab, c->temb_tab,
                   c->cs_all, c->cs_need, c->bmodtab, c->fmodtab, c->dsums, c->vws, c->g_lat, c->g_cond,
-                  c->h_latent, c->h_cond};
+                  c->h_latent, c->h_cond, c->d_rmask, c->d_cmask};
   for (void* p : bufs)
     if (p) cudaFree(p);
   for (int k = 0; k < NKCLASS; ++k)
@@ -1181,6 +1188,37 @@ featfix_status featfix_set_schedule(featfix_ctx* ctx, int steps, const int* refr
   ctx->next_step = 0;
   ctx->cnt = {0, 0, 0, 0};
   ctx->log_sites.clear();
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_set_forward_mask(featfix_ctx* ctx, int axis, const unsigned char* mask, int n) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (axis == FEATFIX_MASK_NONE) {
+    if (ctx->fmask_axis != FEATFIX_MASK_NONE) graph_reset(ctx);
+    ctx->fmask_axis = FEATFIX_MASK_NONE;
+    return FEATFIX_OK;
+  }
+  if (axis != FEATFIX_MASK_TOKENS && axis != FEATFIX_MASK_CHANNELS) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "unknown mask axis");
+  if (!mask) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "null mask");
+  const int want = axis == FEATFIX_MASK_TOKENS ? ctx->Nt + ctx->Ni : ctx->C;
+  if (n != want) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "mask length " + std::to_string(n) + ", expected " + std::to_string(want));
+  FF_CK(cudaStreamSynchronize(ctx->user_st));
+  graph_reset(ctx);
+  std::vector<unsigned char> h;
+  unsigned char** dst;
+  if (axis == FEATFIX_MASK_TOKENS) {  // per token row of every model sample
+    h.assign((size_t)ctx->T, 0);
+    for (int b = 0; b < ctx->Bm; ++b)
+      for (int t = 0; t < n; ++t) h[(size_t)featfix_token_row(&ctx->d, b, t)] = mask[t] ? 1 : 0;
+    dst = &ctx->d_rmask;
+  } else {
+    h.assign(mask, mask + n);
+    for (auto& v : h) v = v ? 1 : 0;
+    dst = &ctx->d_cmask;
+  }
+  if (!*dst) FF_TRY(alloc(ctx, (void**)dst, h.size()));
+  FF_CK(cudaMemcpy(*dst, h.data(), h.size(), cudaMemcpyHostToDevice));
+  ctx->fmask_axis = axis;
   return FEATFIX_OK;
 }
 

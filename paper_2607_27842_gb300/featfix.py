@@ -23,6 +23,7 @@ PLAN_EXACT, PLAN_DRAFT, PLAN_SITE = 0, 1, 2
 FLAG_TAYLOR_RECURSIVE = 1
 FLAG_PER_BLOCK_DRAFT = 2
 FLAG_SITE_UPDATES_HISTORY = 4
+MASK_NONE, MASK_TOKENS, MASK_CHANNELS = 0, 1, 2
 KCLASS = {"gemm": 0, "attention": 1, "draft": 2, "verify": 3, "other": 4}
 
 
@@ -72,6 +73,7 @@ SIGNATURES = {
     "featfix_get_plan": (_I, [_VP, _P(ctypes.c_ubyte), _P(_I), _P(_D)]),
     "featfix_plan_build": (_I, [_I, _I, _P(_I), _I, _I, _P(Site), _I, _I, ctypes.c_uint, _P(ctypes.c_ubyte),
                                 _P(_I), _P(_D)]),
+    "featfix_set_forward_mask": (_I, [_VP, _I, _P(ctypes.c_ubyte), _I]),
     "featfix_plan_build_blocks": (_I, [_I, _I, _P(_I), _I, _I, _P(Site), _I, _I, ctypes.c_uint, _P(_I), _P(_D)]),
     "featfix_debug_capture": (_I, [_VP, _I, _I, _VP, _VP]),
     "featfix_debug_block": (_I, [_VP, _I, _I, _VP, _VP, _VP]),
@@ -269,6 +271,17 @@ def featfix_get_plan(ctx, steps, n_layers):
     return kinds.reshape(steps, n_layers), keff, w.reshape(steps, 4)
 
 
+def featfix_set_forward_mask(ctx, axis, mask=None):
+    """Partial forwarding at FeatFix sites: axis MASK_TOKENS / MASK_CHANNELS
+    with a 0/1 mask, or MASK_NONE (whole-block forwarding)."""
+    import numpy as np
+    if mask is None:
+        _check(lib().featfix_set_forward_mask(ctx, int(axis), None, 0), ctx)
+        return
+    m = np.ascontiguousarray(np.asarray(mask, dtype=np.uint8))
+    _check(lib().featfix_set_forward_mask(ctx, int(axis), m.ctypes.data_as(_P(ctypes.c_ubyte)), int(m.size)), ctx)
+
+
 def featfix_plan_build_blocks(steps, n_layers, refresh, draft_order, sites, mode="featfix", flags=0):
     """Host-only per-block draft plan: (k_eff [steps, L], weights [steps, L, 4])."""
     import numpy as np
@@ -295,6 +308,17 @@ def featfix_plan_build(steps, n_layers, refresh, draft_order, sites, mode="featf
                                     int(flags), kinds.ctypes.data_as(_P(ctypes.c_ubyte)),
                                     keff.ctypes.data_as(_P(_I)), w.ctypes.data_as(_P(_D))))
     return kinds.reshape(steps, n_layers), keff, w.reshape(steps, 4)
+
+
+def featfix_set_forward_mask(ctx, axis, mask=None):
+    """Partial forwarding at FeatFix sites: axis MASK_TOKENS / MASK_CHANNELS
+    with a 0/1 mask, or MASK_NONE (whole-block forwarding)."""
+    import numpy as np
+    if mask is None:
+        _check(lib().featfix_set_forward_mask(ctx, int(axis), None, 0), ctx)
+        return
+    m = np.ascontiguousarray(np.asarray(mask, dtype=np.uint8))
+    _check(lib().featfix_set_forward_mask(ctx, int(axis), m.ctypes.data_as(_P(ctypes.c_ubyte)), int(m.size)), ctx)
 
 
 def featfix_plan_build_blocks(steps, n_layers, refresh, draft_order, sites, mode="featfix", flags=0):

@@ -124,8 +124,18 @@ SHAPES = {
 }
 
 
+# FLUX at lower resolutions (latent 64x64 / 96x96 for 512^2 / 768^2 images,
+# 1024 / 2304 image tokens) with the FLUX schedule: the resolution sweep.
+RESOLUTIONS = {"flux_512": 64, "flux_768": 96}
+
+
 def workload(name):
     """The schedule of each workload: draft order, refresh interval, sites."""
+    if name in RESOLUTIONS:
+        base = workload("flux")
+        side = RESOLUTIONS[name]
+        return Workload(reduced(base.shape, name=name, lat_h=side, lat_w=side), base.steps, base.K, base.refresh,
+                        base.sites)
     s = SHAPES[name]
     if name == "tiny":
         return Workload(s, 10, 1, (0, 3, 6, 9), ((4, 2), (7, 1)))

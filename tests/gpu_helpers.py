@@ -97,12 +97,13 @@ class Case:
         out[self.rows().reshape(-1)] = np.asarray(arr).reshape(-1, sh.hidden)
         return torch.from_numpy(out).to(syn.torch_dtype(sh)).to(self.dev)
 
-    def oracle_run(self, mode="featfix", seed=1, refresh=None, sites=None, hook=None, site_updates_history=False):
+    def oracle_run(self, mode="featfix", seed=1, refresh=None, sites=None, hook=None, site_updates_history=False,
+                   forward_mask=None):
         wl = self.wl
         return oracle.featfix.run(self.W64, self.sh, self.cond64, oracle.noise.initial_latent(seed, self.sh),
                                   wl.steps, wl.refresh if refresh is None else refresh, wl.K,
                                   wl.sites if sites is None else sites, mode, hook=hook,
-                                  site_updates_history=site_updates_history)
+                                  site_updates_history=site_updates_history, forward_mask=forward_mask)
 
     def close(self):
         ff.featfix_destroy(self.ctx)

@@ -98,6 +98,41 @@ def test_site_history_push_matches_oracle(case, mode):
     assert np.abs(x_ref - x_def).max() > 0
 
 
+@pytest.mark.parametrize("axis", ["tokens", "channels"])
+def test_partial_forwarding_matches_oracle(case, axis):
+    """Token / channel partial forwarding at FeatFix sites against the
+    oracle; the all-selected mask is FeatFix bitwise and the none-selected
+    mask is the per-block Verify trajectory bitwise."""
+    n = case.sh.tokens if axis == "tokens" else case.sh.hidden
+    ax = ff.MASK_TOKENS if axis == "tokens" else ff.MASK_CHANNELS
+    mask = (np.arange(n) % 3 == 0).astype(np.uint8)
+    case.schedule("featfix")
+    ff.featfix_set_forward_mask(case.ctx, ax, mask)
+    lat = case.sample(seed=1)
+    x_ref, _, cnt_ref = case.oracle_run("featfix", seed=1, forward_mask=(axis, mask))
+    err = rel_l2(lat.cpu().numpy(), x_ref)
+    assert err < tol_latent(case.sh), err
+    _, cnt = ff.featfix_get_log(case.ctx)
+    assert {k: cnt[k] for k in cnt_ref} == cnt_ref
+    ff.featfix_set_forward_mask(case.ctx, ax, np.ones(n, np.uint8))
+    ones = case.sample(seed=1)
+    ff.featfix_set_forward_mask(case.ctx, ff.MASK_NONE)
+    whole = case.sample(seed=1)
+    # per-block drafts in both arms (the default evaluates site-free drafted
+    # steps in one telescoped pass, equal only up to rounding)
+    case.schedule("featfix", flags=ff.FLAG_PER_BLOCK_DRAFT)
+    ff.featfix_set_forward_mask(case.ctx, ax, np.zeros(n, np.uint8))
+    zeros = case.sample(seed=1)
+    ff.featfix_set_forward_mask(case.ctx, ff.MASK_NONE)
+    case.schedule("verify", flags=ff.FLAG_PER_BLOCK_DRAFT)
+    verify = case.sample(seed=1)
+    assert torch.equal(ones, whole)
+    assert torch.equal(zeros, verify)
+    assert not torch.equal(lat, whole) and not torch.equal(lat, verify)
+    with pytest.raises(ff.FeatFixError):
+        ff.featfix_set_forward_mask(case.ctx, ax, np.ones(n + 1, np.uint8))
+
+
 def test_blocks_teacher_forced(case):
     """Every block of the trajectory on the GPU's own incoming state: exact
     blocks vs B_l (Eq. 1), drafts vs Eq. 2 over the GPU's refresh increments."""

@@ -556,6 +556,34 @@ def test_site_history_push_reading():
     assert logs[0]["rel_l1"] == base[0]["rel_l1"]
 
 
+def test_partial_forwarding_arms_reduce_to_the_whole_block_arms():
+    """Token / channel partial forwarding: all selected = FeatFix, none
+    selected = the draft (Verify's forward), and a mixed mask forwards h_f
+    exactly on the selected tokens / channels of each site."""
+    wl, sh, W, cond, xT = tiny_setup()
+    args = (W, sh, cond, xT, wl.steps, wl.refresh, wl.K, wl.sites)
+    ff_x, _, _ = featfix.run(*args, "featfix")
+    vf_x, _, _ = featfix.run(*args, "verify")
+    n_tok, C = sh.tokens, sh.hidden
+    for axis, n in (("tokens", n_tok), ("channels", C)):
+        a, _, _ = featfix.run(*args, "featfix", forward_mask=(axis, np.ones(n)))
+        np.testing.assert_array_equal(a, ff_x)
+        b, _, _ = featfix.run(*args, "featfix", forward_mask=(axis, np.zeros(n)))
+        np.testing.assert_array_equal(b, vf_x)
+        m = (np.arange(n) % 3) == 0
+        seen = []
+        def hook(i, l, kind, u, h, extra):
+            if kind == schedule.SITE:
+                sel = m[None, :, None] if axis == "tokens" else m[None, None, :]
+                sel = np.broadcast_to(sel, h.shape)
+                np.testing.assert_array_equal(h[sel], extra["h_f"][sel])
+                np.testing.assert_array_equal(h[~sel], extra["h_d"][~sel])
+                seen.append((i, l))
+        c, _, _ = featfix.run(*args, "featfix", hook=hook, forward_mask=(axis, m))
+        assert seen == sorted(wl.sites)
+        assert np.abs(c - ff_x).max() > 0 and np.abs(c - vf_x).max() > 0
+
+
 def test_discrepancy_definitions():
     hf = np.array([1.0, -2.0, 3.0])
     hd = np.array([1.5, -2.0, 2.0])
