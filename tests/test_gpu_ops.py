@@ -50,8 +50,8 @@ def test_draft_exact_on_polynomial_increments(cuda, K):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_draft_matches_oracle(cuda, dtype):
-    n = 5 * 8192 + 24
+@pytest.mark.parametrize("n", [5 * 8192 + 24, 29831168 + 24])   # small; HunyuanVideo's E (tensors > L2) + tail
+def test_draft_matches_oracle(cuda, dtype, n):
     s = [18, 12, 6]
     hist = [randn(n, dtype, 10 + j, 0.05) for j in range(3)]
     x = randn(n, dtype, 3)
@@ -69,7 +69,7 @@ def test_draft_matches_oracle(cuda, dtype):
 # ----------------------------------------------------------------------------
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("n", [1000, 4718592 + 8])
+@pytest.mark.parametrize("n", [1000, 4718592 + 8, 29831168 + 8])   # tiny, DiT-XL/2's E, HunyuanVideo's E
 def test_verify_sums_and_forwarding(cuda, dtype, n):
     hist = [randn(n, dtype, 20 + j, 0.05) for j in range(2)]
     w = [1.4, -0.4]
