@@ -1,7 +1,9 @@
 // Non-causal attention softmax(q k^T / sqrt(d)) v of the exact block (Eq. 1)
 // on the 5th-generation tensor cores, bf16 in, fp32 accumulate.
 //
-// One CTA per (sample, head, pair of 128-query tiles), 10 warps:
+// One CTA per (sample, head, pair of 128-query tiles), 10 warps (sequences
+// of at most four key tiles: one query tile per CTA, 6 warps, two CTAs per
+// SM):
 //   warp 0     TMA producer: both query tiles once, then key and value tiles
 //              of 128 tokens into separate rings, straight from the fused qkv
 //              activation (3-D tensor map: head width, head slot, row; the
@@ -17,7 +19,8 @@
 //              sum, P as bf16 pairs back into TMEM; O is rescaled in TMEM only
 //              when the running max grew by more than 2^8 (the final division
 //              uses the same stale max, so the result is unchanged).
-// TMEM columns: S_0 [0,128), S_1 [128,256), O_0 [256,384), O_1 [384,512).
+// TMEM columns: S_0 [0,128), S_1 [128,256), O_0 [256,384), O_1 [384,512);
+// with one query tile per CTA (short sequences): S [0,128), O [128,256).
 // Keys of a sample lie in up to two row segments (text rows, image rows of
 // the stream-major token layout); tiles never straddle a segment and keys
 // past a segment's end are masked.
@@ -38,8 +41,8 @@ using namespace tc;
 
 constexpr int AQ = 128;        // queries per tile (MMA M)
 constexpr int AKV = 128;       // keys per tile (MMA N of S, K of P V)
-constexpr int ATHREADS = 320;
 constexpr float RESCALE_LOG2 = 8.0f;
+constexpr int SHORT_KV_TILES = 4;  // sequences of at most 4 x 128 tokens: one query tile per CTA
 constexpr size_t SMEM_LIMIT = 232448;  // opt-in dynamic shared memory per block
 
 __device__ unsigned int g_attn_watchdog;
@@ -50,23 +53,30 @@ __device__ __forceinline__ bool wait_a(uint64_t* b, uint32_t parity, volatile in
   return mbar_wait<true>(b, parity, abort_flag, &g_attn_watchdog);
 }
 
-template <int D> struct ACfg {
+// QT query tiles per CTA.  QT = 2: two softmax warpgroups that overlap
+// each other's MMAs, key / value rings as deep as shared memory allows, one
+// CTA per SM.  QT = 1 (short sequences, a couple of key tiles): one softmax
+// warpgroup, single-slot rings and half the TMEM, so two CTAs share an SM
+// and overlap their latency chains instead.
+template <int D, int QT> struct ACfg {
+  static constexpr int THREADS = 64 + 128 * QT;          // TMA warp, MMA warp, softmax warpgroups
   static constexpr int NBOX = D <= 64 ? 1 : 2;           // 64-wide column boxes per tile row
   static constexpr int DK = (D + 15) / 16 * 16;          // q k^T reduction width and P V output width
   static constexpr uint32_t BOX = 128 * 128;             // one [128 rows x 64] bf16 box, 16 KB
   static constexpr uint32_t TILE = NBOX * BOX;           // one Q, K or V tile
-  static constexpr int NST = (int)((SMEM_LIMIT - 1024 - 512 - 2 * (size_t)TILE) / TILE);
-  static constexpr int KST = NST >= 8 ? 4 : (NST + 1) / 2;  // key ring depth
-  static constexpr int VST = NST >= 8 ? 4 : NST / 2;        // value ring depth
-  static constexpr size_t SMEM = 1024 + (size_t)(2 + KST + VST) * TILE + 512;
-  static constexpr uint32_t TMEM_O = 2 * AKV;
+  static constexpr int NST = (int)((SMEM_LIMIT - 1024 - 512 - QT * (size_t)TILE) / TILE);
+  static constexpr int KST = QT == 1 ? 1 : NST >= 8 ? 4 : (NST + 1) / 2;  // key ring depth
+  static constexpr int VST = QT == 1 ? 1 : NST >= 8 ? 4 : NST / 2;        // value ring depth
+  static constexpr size_t SMEM = 1024 + (size_t)(QT + KST + VST) * TILE + 512;
+  static constexpr uint32_t TMEM_O = QT * AKV;           // S_i at i * 128, O_i at TMEM_O + i * 128
+  static constexpr uint32_t TMEM_COLS = QT == 1 ? 256 : 512;
   // kind::f16, D fp32, A/B bf16; S: both K-major, N = 128; O: A (P) from
   // TMEM, B (V) MN-major (bit 16), N = DK
   static constexpr uint32_t IDESC_S = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(AKV >> 3) << 17) |
                                       ((uint32_t)(AQ >> 4) << 24);
   static constexpr uint32_t IDESC_O = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((uint32_t)(DK >> 3) << 17) |
                                       ((uint32_t)(AQ >> 4) << 24);
-  static_assert(KST >= 2 && VST >= 1, "shared memory too small for the key/value rings");
+  static_assert(KST >= 1 && VST >= 1 && (QT == 1 || KST >= 2), "shared memory too small for the key/value rings");
   static_assert(SMEM <= SMEM_LIMIT, "shared memory budget");
 };
 
@@ -147,14 +157,14 @@ __device__ __forceinline__ SegTile seg_tile(const AttnArgs& a, int b, int t) {
   return {a.B * a.Nt + b * a.Ni + u * 128, min(128, a.Ni - u * 128)};
 }
 
-template <int D>
-__global__ void __launch_bounds__(ATHREADS, 1)
+template <int D, int QT>
+__global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
     k_attn_tc(const __grid_constant__ CUtensorMap tmQKV, AttnArgs a, float scale_log2) {
-  using C = ACfg<D>;
+  using C = ACfg<D, QT>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQ = smem;                        // 2 tiles
-  uint8_t* sK = sQ + 2 * C::TILE;            // KST tiles
+  uint8_t* sQ = smem;                        // QT tiles
+  uint8_t* sK = sQ + QT * C::TILE;           // KST tiles
   uint8_t* sV = sK + C::KST * C::TILE;       // VST tiles
   uint64_t* bars = reinterpret_cast<uint64_t*>(sV + C::VST * C::TILE);
   uint64_t* q_full = bars;
@@ -182,7 +192,7 @@ __global__ void __launch_bounds__(ATHREADS, 1)
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < QT; ++i) {
       mbar_init(&s_full[i], 1);
       mbar_init(&p_ready[i], 128);
     }
@@ -192,7 +202,8 @@ __global__ void __launch_bounds__(ATHREADS, 1)
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQKV) : "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(tmem_slot)), "r"(512)
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(tmem_slot)),
+                 "r"(C::TMEM_COLS)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -207,9 +218,9 @@ __global__ void __launch_bounds__(ATHREADS, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      mbar_expect_tx(q_full, 2 * C::TILE);
-      for (int i = 0; i < 2; ++i) {
-        const SegTile qs = seg_tile(a, b, 2 * blockIdx.x + i);
+      mbar_expect_tx(q_full, QT * C::TILE);
+      for (int i = 0; i < QT; ++i) {
+        const SegTile qs = seg_tile(a, b, QT * blockIdx.x + i);
         for (int bx = 0; bx < C::NBOX; ++bx) tma_load3(&tmQKV, q_full, sQ + i * C::TILE + bx * C::BOX, 64 * bx, h, qs.row0);
       }
       int nk = 0, nv = 0;
@@ -262,14 +273,14 @@ __global__ void __launch_bounds__(ATHREADS, 1)
       if (ok) {
         tc_fence_after();
         issue_s(0, 0);
-        issue_s(1, 0);
+        if (QT == 2) issue_s(1, 0);
         umma_commit(&k_empty[0]);
       }
       for (int j = 0; j < nkv && ok; ++j) {
         const int sv = j % C::VST;
         if (!wait_a(&v_full[sv], (j / C::VST) & 1, abort_flag)) break;
         const uint32_t vaddr = saddr(sV + sv * C::TILE);
-        for (int i = 0; i < 2 && ok; ++i) {
+        for (int i = 0; i < QT && ok; ++i) {
           if (!wait_a(&p_ready[i], j & 1, abort_flag)) { ok = false; break; }
           tc_fence_after();
           // O_i += P_i V_j: 16 keys per step = 8 TMEM columns of P, 2 groups
@@ -286,7 +297,7 @@ __global__ void __launch_bounds__(ATHREADS, 1)
               tc_fence_after();
             }
             issue_s(i, j + 1);  // behind O_i's update: the MMA pipe reads P_i before S_i is overwritten
-            if (i == 1) umma_commit(&k_empty[(j + 1) % C::KST]);
+            if (i == QT - 1) umma_commit(&k_empty[(j + 1) % C::KST]);
           }
         }
         if (!ok) break;
@@ -302,7 +313,7 @@ __global__ void __launch_bounds__(ATHREADS, 1)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const uint32_t s_col = tmem + lane_off + (uint32_t)(i * AKV);
     const uint32_t o_col = tmem + lane_off + C::TMEM_O + (uint32_t)(i * AKV);
-    const SegTile qs = seg_tile(a, b, 2 * blockIdx.x + i);
+    const SegTile qs = seg_tile(a, b, QT * blockIdx.x + i);
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nkv; ++j) {
@@ -406,7 +417,7 @@ __global__ void __launch_bounds__(ATHREADS, 1)
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TMEM_COLS) : "memory");
   }
 }
 
@@ -420,9 +431,10 @@ bool init_attn() {
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
       g_enc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    cudaFuncSetAttribute(k_attn_tc<72>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ACfg<72>::SMEM);
-    cudaFuncSetAttribute(k_attn_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ACfg<128>::SMEM);
-    cudaFuncSetAttribute(k_attn_tc<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ACfg<64>::SMEM);
+#define FF_ATTR(d, qt) \
+  cudaFuncSetAttribute(k_attn_tc<d, qt>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ACfg<d, qt>::SMEM)
+    FF_ATTR(64, 1); FF_ATTR(64, 2); FF_ATTR(72, 1); FF_ATTR(72, 2); FF_ATTR(128, 1); FF_ATTR(128, 2);
+#undef FF_ATTR
   });
   return g_enc != nullptr;
 }
@@ -442,10 +454,16 @@ cudaError_t attn_tc_t(const AttnArgs& a, cudaStream_t s) {
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return cudaErrorInvalidValue;
-  const int nq = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;  // query tiles per sample, two per CTA
-  dim3 grid((nq + 1) / 2, a.H, a.B);
+  // query tiles per sample; short sequences (a few key tiles) run one query
+  // tile per CTA, two CTAs per SM, longer ones two query tiles per CTA
+  const int nq = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)D);
-  launch_pdl(k_attn_tc<D>, grid, ATHREADS, ACfg<D>::SMEM, s, tm, a, scale_log2);
+  if (nq <= SHORT_KV_TILES) {
+    launch_pdl(k_attn_tc<D, 1>, dim3(nq, a.H, a.B), ACfg<D, 1>::THREADS, ACfg<D, 1>::SMEM, s, tm, a, scale_log2);
+  } else {
+    launch_pdl(k_attn_tc<D, 2>, dim3((nq + 1) / 2, a.H, a.B), ACfg<D, 2>::THREADS, ACfg<D, 2>::SMEM, s, tm, a,
+               scale_log2);
+  }
   return launched();
 }
 
