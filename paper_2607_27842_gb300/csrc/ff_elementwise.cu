@@ -286,14 +286,31 @@ cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int
 // One warp per row, the row held in registers (NCH 16-byte vectors per
 // lane): one global read, exact two-pass mean / variance, one write.
 // ---------------------------------------------------------------------------
+// One warp per row (8 rows per block); the block first stages the shift /
+// scale vectors of its first row's sample in shared memory (coalesced, read
+// back by every warp of that sample instead of 4 x 16 B per lane per chunk
+// from global memory).
 template <class T, int NCH>
 __global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
                                                 const float* __restrict__ shift, const float* __restrict__ scale,
                                                 int mod_stride, int seg_split, int rpb0, int rpb1) {
   pdl_trigger();
   pdl_wait();
+  extern __shared__ float4 smod4[];                  // [2 * C / 4]: shift, then scale
+  float* smod = reinterpret_cast<float*>(smod4);
   constexpr int V = VecN<T>::n;
-  const long long r = (long long)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const long long r0 = (long long)blockIdx.x * 8;
+  const int b0 = (int)(r0 < seg_split ? r0 / rpb0 : (r0 - seg_split) / rpb1);
+  {
+    const float4* sh4 = reinterpret_cast<const float4*>(shift + (size_t)b0 * mod_stride);
+    const float4* sc4 = reinterpret_cast<const float4*>(scale + (size_t)b0 * mod_stride);
+    for (int i = threadIdx.x; i < C / 4; i += blockDim.x) {
+      smod4[i] = sh4[i];
+      smod4[C / 4 + i] = sc4[i];
+    }
+  }
+  __syncthreads();
+  const long long r = r0 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
   const T* xr = x + r * C;
@@ -322,8 +339,10 @@ __global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __re
   ss = warp_sum(ss);
   const float rstd = rsqrtf(ss / C + 1e-6f);
   const int b = (int)(r < seg_split ? r / rpb0 : (r - seg_split) / rpb1);
-  const float* sh = shift + (size_t)b * mod_stride;
-  const float* sc = scale + (size_t)b * mod_stride;
+  // the block's sample from shared memory, a second sample (a block straddling
+  // a sample boundary) from global memory
+  const float* sh = b == b0 ? smod : shift + (size_t)b * mod_stride;
+  const float* sc = b == b0 ? smod + C : scale + (size_t)b * mod_stride;
   T* orow = out + r * C;
 #pragma unroll
   for (int j = 0; j < NCH; ++j) {
@@ -350,17 +369,19 @@ static cudaError_t ln_mod_t(const void* x, void* out, long long rows, int C, con
   constexpr int V = VecN<T>::n;
   const int nch = (C / V + 31) / 32;
   const unsigned grid = (unsigned)((rows + 7) / 8);
+  const size_t smem = (size_t)2 * C * sizeof(float);  // shift + scale of one sample
+  if (C % 4 != 0 || smem > 48 * 1024) return cudaErrorInvalidValue;
   const T* xp = (const T*)x;
   T* op = (T*)out;
 #define FF_LN_CASE(n) \
-  case n: launch_pdl(k_ln_mod<T, n>, grid, 256, 0, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break;
+  case n: launch_pdl(k_ln_mod<T, n>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break;
   switch (nch) {
     FF_LN_CASE(1) FF_LN_CASE(2) FF_LN_CASE(3) FF_LN_CASE(4) FF_LN_CASE(5) FF_LN_CASE(6)
     FF_LN_CASE(8) FF_LN_CASE(12) FF_LN_CASE(16)
     default:
-      if (nch <= 8) { launch_pdl(k_ln_mod<T, 8>, grid, 256, 0, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
-      if (nch <= 12) { launch_pdl(k_ln_mod<T, 12>, grid, 256, 0, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
-      if (nch <= 16) { launch_pdl(k_ln_mod<T, 16>, grid, 256, 0, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      if (nch <= 8) { launch_pdl(k_ln_mod<T, 8>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      if (nch <= 12) { launch_pdl(k_ln_mod<T, 12>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
+      if (nch <= 16) { launch_pdl(k_ln_mod<T, 16>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
       return cudaErrorInvalidValue;
   }
 #undef FF_LN_CASE
