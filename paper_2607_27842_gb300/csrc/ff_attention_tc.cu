@@ -8,17 +8,23 @@
 //              of 128 tokens into separate rings, straight from the fused qkv
 //              activation (3-D tensor map: head width, head slot, row; the
 //              head width is zero-padded to a multiple of 64 by the map);
-//   warp 1     TMEM allocator and MMA issuer.  Per key tile j and query tile
-//              i: S_i = Q_i K_j^T into TMEM (both operands K-major from shared
+//   warp 1     TMEM allocator and MMA issuer (the whole warp runs the loop,
+//              one elected lane issues).  Per key tile j and query tile i:
+//              S_i = Q_i K_j^T into TMEM (both operands K-major from shared
 //              memory), then O_i += P_i V_j with P_i read from TMEM (where the
 //              softmax wrote it over S_i) and V MN-major from its TMA tile.
 //              S_i for tile j + 1 is issued right behind O_i's update for
-//              tile j, so one query tile's softmax overlaps the other's MMAs;
+//              tile j, so one query tile's softmax overlaps the other's MMAs.
+//              The issuing thread runs only a few MMAs ahead of the tensor
+//              pipe, so every gap between two groups of MMAs holds at most
+//              one barrier wait;
 //   warps 2-5  softmax of query tile 0, warps 6-9 of query tile 1: each
-//              thread owns one query row (its TMEM lane): row max, exp2, row
-//              sum, P as bf16 pairs back into TMEM; O is rescaled in TMEM only
-//              when the running max grew by more than 2^8 (the final division
-//              uses the same stale max, so the result is unchanged).
+//              thread owns one query row (its TMEM lane): row max, exp2,
+//              row sum, P as bf16 pairs back into TMEM; O is rescaled in TMEM
+//              only when the running max grew by more than 2^8 (the final
+//              division uses the same stale max, so the result is unchanged).
+//              The two warpgroups take turns (a token barrier) so that one
+//              tile's softmax runs while the tensor pipe works on the other.
 // TMEM columns: S_0 [0,128), S_1 [128,256), O_0 [256,384), O_1 [384,512);
 // with one query tile per CTA (short sequences): S [0,128), O [128,256).
 // Keys of a sample lie in up to two row segments (text rows, image rows of
@@ -52,6 +58,12 @@ __device__ unsigned int g_attn_watchdog;
 __device__ __forceinline__ bool wait_a(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
   return mbar_wait<true>(b, parity, abort_flag, &g_attn_watchdog);
 }
+// the MMA warp's waits: every lane polls, the vote makes the outcome (and so
+// the loop control and the operand descriptors behind it) warp-uniform
+__device__ __forceinline__ bool wait_u(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
+  const bool ok = mbar_test(b, parity) || wait_a(b, parity, abort_flag);
+  return __all_sync(0xffffffffu, ok);
+}
 
 // QT query tiles per CTA.  QT = 2: two softmax warpgroups that overlap
 // each other's MMAs, key / value rings as deep as shared memory allows, one
@@ -59,7 +71,8 @@ __device__ __forceinline__ bool wait_a(uint64_t* b, uint32_t parity, volatile in
 // warpgroup, single-slot rings and half the TMEM, so two CTAs share an SM
 // and overlap their latency chains instead.
 template <int D, int QT> struct ACfg {
-  static constexpr int THREADS = 64 + 128 * QT;          // TMA warp, MMA warp, softmax warpgroups
+  static constexpr int SOFT_WARP0 = 2;                   // first softmax warp
+  static constexpr int THREADS = 32 * SOFT_WARP0 + 128 * QT;  // TMA warp, MMA warp, softmax warpgroups
   static constexpr int NBOX = D <= 64 ? 1 : 2;           // 64-wide column boxes per tile row
   static constexpr int DK = (D + 15) / 16 * 16;          // q k^T reduction width and P V output width
   static constexpr uint32_t BOX = 128 * 128;             // one [128 rows x 64] bf16 box, 16 KB
@@ -104,18 +117,13 @@ __device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64
 
 // 64 consecutive 32-bit TMEM columns of this warp's 32 lanes, waited for in
 // the same statement so no use of the registers can precede the wait
-__device__ __forceinline__ void tmem_ld64w(uint32_t taddr, uint32_t (&r)[64]) {
+// 64 consecutive 32-bit TMEM columns of this warp's 32 lanes, waited for in
+// the same statement so no use of the registers can precede the wait
+__device__ __forceinline__ void tmem_ld64w(uint32_t taddr, float* v) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];\n"
       "tcgen05.wait::ld.sync.aligned;\n"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
-        "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]),
-        "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]),
-        "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
-        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]), "=f"(v[7]), "=f"(v[8]), "=f"(v[9]), "=f"(v[10]), "=f"(v[11]), "=f"(v[12]), "=f"(v[13]), "=f"(v[14]), "=f"(v[15]), "=f"(v[16]), "=f"(v[17]), "=f"(v[18]), "=f"(v[19]), "=f"(v[20]), "=f"(v[21]), "=f"(v[22]), "=f"(v[23]), "=f"(v[24]), "=f"(v[25]), "=f"(v[26]), "=f"(v[27]), "=f"(v[28]), "=f"(v[29]), "=f"(v[30]), "=f"(v[31]), "=f"(v[32]), "=f"(v[33]), "=f"(v[34]), "=f"(v[35]), "=f"(v[36]), "=f"(v[37]), "=f"(v[38]), "=f"(v[39]), "=f"(v[40]), "=f"(v[41]), "=f"(v[42]), "=f"(v[43]), "=f"(v[44]), "=f"(v[45]), "=f"(v[46]), "=f"(v[47]), "=f"(v[48]), "=f"(v[49]), "=f"(v[50]), "=f"(v[51]), "=f"(v[52]), "=f"(v[53]), "=f"(v[54]), "=f"(v[55]), "=f"(v[56]), "=f"(v[57]), "=f"(v[58]), "=f"(v[59]), "=f"(v[60]), "=f"(v[61]), "=f"(v[62]), "=f"(v[63])
       : "r"(taddr)
       : "memory");
 }
@@ -175,7 +183,8 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
   uint64_t* s_full = v_empty + C::VST;       // per query tile
   uint64_t* p_ready = s_full + 2;            // per query tile
   uint64_t* o_final = p_ready + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_final + 1);
+  uint64_t* tok = o_final + 1;               // ping-pong token of the two softmax warpgroups
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tok + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -197,6 +206,9 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       mbar_init(&p_ready[i], 128);
     }
     mbar_init(o_final, 1);
+    mbar_init(&tok[0], 4);  // one arrival per warp of the passing warpgroup
+    mbar_init(&tok[1], 4);
+    for (int w = 0; w < 4; ++w) mbar_arrive(&tok[0]);  // warpgroup 0 holds the token first
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQKV) : "memory");
@@ -254,60 +266,63 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      bool ok = wait_a(q_full, 0, abort_flag);
-      const uint64_t qd0 = sw128_desc(saddr(sQ)), qd1 = sw128_desc(saddr(sQ + C::TILE));
-      // S_i = Q_i K_j^T (DK / 16 steps of 16 along the head width: box k / 4,
-      // +32 B per step inside the box), then arrive on s_full[i]
-      auto issue_s = [&](int i, int j) {
-        const uint64_t kd = sw128_desc(saddr(sK + (j % C::KST) * C::TILE));
-        const uint64_t qd = i ? qd1 : qd0;
+    bool ok = wait_u(q_full, 0, abort_flag);
+    const uint64_t qd0 = sw128_desc(saddr(sQ)), qd1 = sw128_desc(saddr(sQ + C::TILE));
+    // S_i = Q_i K_j^T (DK / 16 steps of 16 along the head width: box k / 4,
+    // +32 B per step inside the box), then arrive on s_full[i]
+    auto issue_s = [&](int i, int j) {
+      const uint64_t kd = sw128_desc(saddr(sK + (j % C::KST) * C::TILE));
+      const uint64_t qd = i ? qd1 : qd0;
 #pragma unroll
-        for (int k = 0; k < C::DK / 16; ++k) {
-          const uint64_t off = (uint64_t)((k >> 2) * (C::BOX >> 4) + 2 * (k & 3));
-          umma(tmem + (uint32_t)(i * AKV), qd + off, kd + off, C::IDESC_S, k != 0);
-        }
-        umma_commit(&s_full[i]);
-      };
-      if (ok) ok = wait_a(&k_full[0], 0, abort_flag);
-      if (ok) {
-        tc_fence_after();
-        issue_s(0, 0);
-        if (QT == 2) issue_s(1, 0);
-        umma_commit(&k_empty[0]);
+      for (int k = 0; k < C::DK / 16; ++k) {
+        const uint64_t off = (uint64_t)((k >> 2) * (C::BOX >> 4) + 2 * (k & 3));
+        if (elect_one()) umma(tmem + (uint32_t)(i * AKV), qd + off, kd + off, C::IDESC_S, k != 0);
       }
-      for (int j = 0; j < nkv && ok; ++j) {
-        const int sv = j % C::VST;
-        if (!wait_a(&v_full[sv], (j / C::VST) & 1, abort_flag)) break;
-        const uint32_t vaddr = saddr(sV + sv * C::TILE);
-        for (int i = 0; i < QT && ok; ++i) {
-          if (!wait_a(&p_ready[i], j & 1, abort_flag)) { ok = false; break; }
-          tc_fence_after();
-          // O_i += P_i V_j: 16 keys per step = 8 TMEM columns of P, 2 groups
-          // of 8 value rows (2 KB) of the MN-major V tile
+      if (elect_one()) umma_commit(&s_full[i]);
+    };
+    if (ok) ok = wait_u(&k_full[0], 0, abort_flag);
+    if (ok) {
+      tc_fence_after();
+      issue_s(0, 0);
+      if (QT == 2) issue_s(1, 0);
+      if (elect_one()) umma_commit(&k_empty[0]);
+      ok = wait_u(&v_full[0], 0, abort_flag);
+    }
+    // Per key tile j: [p_ready 0] O_0 += P_0 V_j [k_full j+1] S_0 for j + 1
+    // [p_ready 1] O_1 += P_1 V_j [v_full j+1] S_1 for j + 1 -- one wait in
+    // each gap between MMA groups
+    for (int j = 0; j < nkv && ok; ++j) {
+      const int sv = j % C::VST;
+      const bool more = j + 1 < nkv;
+      const uint32_t vaddr = saddr(sV + sv * C::TILE);
+      for (int i = 0; i < QT; ++i) {
+        ok = wait_u(&p_ready[i], j & 1, abort_flag);
+        if (!ok) break;
+        tc_fence_after();
+        // O_i += P_i V_j: 16 keys per step = 8 TMEM columns of P, 2 groups
+        // of 8 value rows (2 KB) of the MN-major V tile
 #pragma unroll
-          for (int k = 0; k < AKV / 16; ++k) {
-            const uint64_t vd = sw128_desc_mn(vaddr + (uint32_t)k * 2048u, C::BOX);
+        for (int k = 0; k < AKV / 16; ++k) {
+          const uint64_t vd = sw128_desc_mn(vaddr + (uint32_t)k * 2048u, C::BOX);
+          if (elect_one())
             umma_ts(tmem + C::TMEM_O + (uint32_t)(i * AKV), tmem + (uint32_t)(i * AKV + k * 8), vd, C::IDESC_O,
                     (j | k) != 0);
-          }
-          if (j + 1 < nkv) {
-            if (i == 0) {
-              if (!wait_a(&k_full[(j + 1) % C::KST], ((j + 1) / C::KST) & 1, abort_flag)) { ok = false; break; }
-              tc_fence_after();
-            }
-            issue_s(i, j + 1);  // behind O_i's update: the MMA pipe reads P_i before S_i is overwritten
-            if (i == QT - 1) umma_commit(&k_empty[(j + 1) % C::KST]);
-          }
         }
-        if (!ok) break;
-        umma_commit(&v_empty[sv]);
+        if (i == QT - 1 && elect_one()) umma_commit(&v_empty[sv]);
+        if (more) {
+          if (i == 0) ok = wait_u(&k_full[(j + 1) % C::KST], ((j + 1) / C::KST) & 1, abort_flag);
+          if (ok && i == QT - 1) ok = wait_u(&v_full[(j + 1) % C::VST], ((j + 1) / C::VST) & 1, abort_flag);
+          if (!ok) break;
+          tc_fence_after();
+          issue_s(i, j + 1);  // behind O_i's update: the MMA pipe reads P_i before S_i is overwritten
+          if (i == QT - 1 && elect_one()) umma_commit(&k_empty[(j + 1) % C::KST]);
+        }
       }
-      if (ok) umma_commit(o_final);
     }
-  } else {
+    if (ok && elect_one()) umma_commit(o_final);
+  } else if (warp >= C::SOFT_WARP0) {
     // softmax of query tile i: row r of the tile = TMEM lane r
-    const int i = (warp - 2) >> 2;
+    const int i = (warp - C::SOFT_WARP0) >> 2;
     const int q = warp & 3;
     const int r = q * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
@@ -319,19 +334,18 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
     for (int j = 0; j < nkv; ++j) {
       const int valid = seg_tile(a, b, j).valid;
       int w = 1;
-      if (lane == 0) w = wait_a(&s_full[i], j & 1, abort_flag) ? 1 : 0;
+      if (lane == 0) {
+        w = wait_a(&s_full[i], j & 1, abort_flag) ? 1 : 0;
+        // two query tiles: the warpgroups take turns for the exp-heavy part
+        // (they share each sub-partition's SFU), so one tile's softmax runs
+        // while the tensor pipe works on the other tile
+        if (QT == 2 && w) w = wait_a(&tok[i], j & 1, abort_flag) ? 1 : 0;
+      }
       if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
       tc_fence_after();
       float v[AKV];
-      {
-        uint32_t t[64];
-        tmem_ld64w(s_col, t);
-#pragma unroll
-        for (int e = 0; e < 64; ++e) v[e] = __uint_as_float(t[e]);
-        tmem_ld64w(s_col + 64, t);
-#pragma unroll
-        for (int e = 0; e < 64; ++e) v[64 + e] = __uint_as_float(t[e]);
-      }
+      tmem_ld64w(s_col, v);
+      tmem_ld64w(s_col + 64, v + 64);
       if (valid < AKV) {
 #pragma unroll
         for (int e = 0; e < AKV; ++e)
@@ -384,6 +398,10 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       l = l * alpha + (((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7])));
       tmem_st_wait();
       tc_fence_before();
+      if (QT == 2) {  // pass the token: it turns once all four warps have arrived
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tok[i ^ 1]);
+      }
       mbar_arrive(&p_ready[i]);
     }
     if (ok) {
