@@ -43,6 +43,13 @@ __device__ unsigned int g_watchdog;
 __device__ __forceinline__ bool mbar_wait_g(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
   return mbar_wait(b, parity, abort_flag, &g_watchdog);
 }
+// the MMA warp's waits: every lane waits, the vote keeps the loop control
+// (and the descriptors computed under it) warp-uniform, so the elected lane's
+// tcgen05.mma does not block the issuing thread
+__device__ __forceinline__ bool mbar_wait_u(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
+  const bool ok = mbar_test(b, parity) || mbar_wait_g(b, parity, abort_flag);
+  return __all_sync(0xffffffffu, ok);
+}
 
 template <int BN> struct Cfg {
   static constexpr int STAGES = BN >= 256 ? 4 : 6;
@@ -182,33 +189,32 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      uint32_t it = 0;
-      int tc = 0;
-      bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++tc) {
-        const int acc = tc & 1;
-        const uint32_t aph = (tc >> 1) & 1;
-        if (!mbar_wait_g(&tempty[acc], aph ^ 1, abort_flag)) break;
+    // the whole warp runs the loop, one elected lane issues
+    uint32_t it = 0;
+    int tc = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++tc) {
+      const int acc = tc & 1;
+      const uint32_t aph = (tc >> 1) & 1;
+      if (!mbar_wait_u(&tempty[acc], aph ^ 1, abort_flag)) break;
+      tc_fence_after();
+      const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+      for (int kb = 0; kb < num_kb; ++kb, ++it) {
+        const int s = it % C::STAGES;
+        const uint32_t ph = (it / C::STAGES) & 1;
+        if (!mbar_wait_u(&full[s], ph, abort_flag)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
-        for (int kb = 0; kb < num_kb; ++kb, ++it) {
-          const int s = it % C::STAGES;
-          const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait_g(&full[s], ph, abort_flag)) { ok = false; break; }
-          tc_fence_after();
-          const uint64_t ad = sw128_desc(saddr(sA + s * C::A_BYTES));
-          const uint64_t bd = sw128_desc(saddr(sB + s * C::B_BYTES));
+        const uint64_t ad = sw128_desc(saddr(sA + s * C::A_BYTES));
+        const uint64_t bd = sw128_desc(saddr(sB + s * C::B_BYTES));
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {
-            // +32 bytes (16 bf16) along K inside the swizzle atom
-            umma(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), C::IDESC, (kb | k) != 0);
-          }
-          umma_commit(&empty[s]);
+        for (int k = 0; k < BK / 16; ++k) {
+          // +32 bytes (16 bf16) along K inside the swizzle atom
+          if (elect_one()) umma(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), C::IDESC, (kb | k) != 0);
         }
-        if (!ok) break;
-        umma_commit(&tfull[acc]);
+        if (elect_one()) umma_commit(&empty[s]);
       }
+      if (!ok) break;
+      if (elect_one()) umma_commit(&tfull[acc]);
     }
   } else {
     // 8 epilogue warps: TMEM lane quarter q = warp % 4 (the quarter a warp
@@ -501,30 +507,30 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0 && leader) {
+    if (leader) {  // the whole warp runs the loop, one elected lane issues
       uint32_t it = 0;
       int tc = 0;
       bool ok = true;
       for (int tile = pair; tile < num_tiles && ok; tile += npairs, ++tc) {
         const int acc = tc & 1;
         const uint32_t aph = (tc >> 1) & 1;
-        if (!mbar_wait_g(&tempty[acc], aph ^ 1, abort_flag)) break;
+        if (!mbar_wait_u(&tempty[acc], aph ^ 1, abort_flag)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait_g(&full[s], ph, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_u(&full[s], ph, abort_flag)) { ok = false; break; }
           tc_fence_after();
           const uint64_t ad = sw128_desc(saddr(sA + s * C::A_BYTES));
           const uint64_t bd = sw128_desc(saddr(sB + s * C::B_BYTES));
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
-            umma_pair(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), C::IDESC, (kb | k) != 0);
-          umma_commit_pair(&empty[s]);
+            if (elect_one()) umma_pair(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), C::IDESC, (kb | k) != 0);
+          if (elect_one()) umma_commit_pair(&empty[s]);
         }
         if (!ok) break;
-        umma_commit_pair(&tfull[acc]);
+        if (elect_one()) umma_commit_pair(&tfull[acc]);
       }
     }
   } else {
