@@ -117,8 +117,6 @@ __device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64
 
 // 64 consecutive 32-bit TMEM columns of this warp's 32 lanes, waited for in
 // the same statement so no use of the registers can precede the wait
-// 64 consecutive 32-bit TMEM columns of this warp's 32 lanes, waited for in
-// the same statement so no use of the registers can precede the wait
 __device__ __forceinline__ void tmem_ld64w(uint32_t taddr, float* v) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];\n"
@@ -138,6 +136,11 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
 }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -351,16 +354,16 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
         for (int e = 0; e < AKV; ++e)
           if (e >= valid) v[e] = -INFINITY;
       }
-      // row max as a tree (depth 7)
+      // row max as a tree of three-input maxima (72 instructions for 128
+      // values instead of 127)
       float mx[16];
 #pragma unroll
       for (int e = 0; e < 16; ++e)
-        mx[e] = fmaxf(fmaxf(fmaxf(v[e], v[e + 16]), fmaxf(v[e + 32], v[e + 48])),
-                      fmaxf(fmaxf(v[e + 64], v[e + 80]), fmaxf(v[e + 96], v[e + 112])));
+        mx[e] = max3f(max3f(v[e], v[e + 16], v[e + 32]), max3f(v[e + 48], v[e + 64], v[e + 80]),
+                      fmaxf(v[e + 96], v[e + 112]));
 #pragma unroll
-      for (int s = 8; s >= 1; s >>= 1)
-#pragma unroll
-        for (int e = 0; e < s; ++e) mx[e] = fmaxf(mx[e], mx[e + s]);
+      for (int e = 0; e < 5; ++e) mx[e] = max3f(mx[e], mx[e + 5], mx[e + 10]);
+      mx[0] = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[15]), mx[0]);
       const float m_new = fmaxf(m, mx[0] * scale_log2);
       const bool grow = m_new > m + RESCALE_LOG2;  // also true on the first tile
       const float m_use = grow ? m_new : m;

@@ -43,6 +43,12 @@ __device__ unsigned int g_watchdog;
 __device__ __forceinline__ bool mbar_wait_g(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
   return mbar_wait(b, parity, abort_flag, &g_watchdog);
 }
+// the producer's waits for a free stage poll: a suspended wait woke up
+// several hundred cycles after the stage's MMAs completed, and the ring is
+// only four stages deep
+__device__ __forceinline__ bool mbar_wait_p(uint64_t* b, uint32_t parity, volatile int* abort_flag) {
+  return mbar_wait<true>(b, parity, abort_flag, &g_watchdog);
+}
 // the MMA warp's waits: every lane waits, the vote keeps the loop control
 // (and the descriptors computed under it) warp-uniform, so the elected lane's
 // tcgen05.mma does not block the issuing thread
@@ -164,7 +170,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait_g(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_p(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
           mbar_expect_tx(&full[s], C::STAGE_BYTES);
           // normal: A rows -> M side, W rows -> N side; swapped: the reverse.
           // (Each call names its kernel parameter: a tensor map must stay in
@@ -489,7 +495,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
-          if (!mbar_wait_g(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait_p(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
           if (leader) mbar_expect_tx(&full[s], 2 * C::STAGE_BYTES);
           const uint32_t fb = map_to(&full[s], 0);
           tma_load_pair(&tmA, fb, sA + s * C::A_BYTES, kb * BK, mb * 2 * BM + (int)rank * BM);
