@@ -23,8 +23,9 @@
 //              row sum, P as bf16 pairs back into TMEM; O is rescaled in TMEM
 //              only when the running max grew by more than 2^8 (the final
 //              division uses the same stale max, so the result is unchanged).
-//              The two warpgroups take turns (a token barrier) so that one
-//              tile's softmax runs while the tensor pipe works on the other.
+//              The two warpgroups run freely (making them take turns for
+//              the exponentials measured slower once the MMA issue stopped
+//              stalling).
 // TMEM columns: S_0 [0,128), S_1 [128,256), O_0 [256,384), O_1 [384,512);
 // with one query tile per CTA (short sequences): S [0,128), O [128,256).
 // Keys of a sample lie in up to two row segments (text rows, image rows of
@@ -186,8 +187,7 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
   uint64_t* s_full = v_empty + C::VST;       // per query tile
   uint64_t* p_ready = s_full + 2;            // per query tile
   uint64_t* o_final = p_ready + 2;
-  uint64_t* tok = o_final + 1;               // ping-pong token of the two softmax warpgroups
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tok + 2);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_final + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -209,9 +209,6 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       mbar_init(&p_ready[i], 128);
     }
     mbar_init(o_final, 1);
-    mbar_init(&tok[0], 4);  // one arrival per warp of the passing warpgroup
-    mbar_init(&tok[1], 4);
-    for (int w = 0; w < 4; ++w) mbar_arrive(&tok[0]);  // warpgroup 0 holds the token first
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQKV) : "memory");
@@ -337,13 +334,7 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
     for (int j = 0; j < nkv; ++j) {
       const int valid = seg_tile(a, b, j).valid;
       int w = 1;
-      if (lane == 0) {
-        w = wait_a(&s_full[i], j & 1, abort_flag) ? 1 : 0;
-        // two query tiles: the warpgroups take turns for the exp-heavy part
-        // (they share each sub-partition's SFU), so one tile's softmax runs
-        // while the tensor pipe works on the other tile
-        if (QT == 2 && w) w = wait_a(&tok[i], j & 1, abort_flag) ? 1 : 0;
-      }
+      if (lane == 0) w = wait_a(&s_full[i], j & 1, abort_flag) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
       tc_fence_after();
       float v[AKV];
@@ -401,10 +392,6 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       l = l * alpha + (((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7])));
       tmem_st_wait();
       tc_fence_before();
-      if (QT == 2) {  // pass the token: it turns once all four warps have arrived
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&tok[i ^ 1]);
-      }
       mbar_arrive(&p_ready[i]);
     }
     if (ok) {
