@@ -83,6 +83,10 @@ struct TileMap {
   int num_m2;  // 256-row blocks of A (swapped tiles)
   int n_tiles; // n_norm + swapped tiles
   int staged;  // normal tiles store out (and hist_out) through shared memory + TMA
+  // one tile per CTA (the TMA ring is idle after its mainloop): each
+  // epilogue warp loads its residual (bit 0) and history-base (bit 1) block
+  // with TMA into the freed ring instead of per-lane global loads
+  int pre;
 };
 
 // 64-byte-swizzled [32 rows x 32 bf16] block: 16-byte chunk k of row r
@@ -109,7 +113,8 @@ template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmW128, const __grid_constant__ CUtensorMap tmA256,
-              const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmH, int M, int N, int K,
+              const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmH,
+              const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmHB, int M, int N, int K,
               TileMap tm, EpiArgs e) {
   using C = Cfg<BN>;
   extern __shared__ uint8_t smem_raw[];
@@ -121,7 +126,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint64_t* empty = full + C::STAGES;
   uint64_t* tfull = empty + C::STAGES;
   uint64_t* tempty = tfull + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  uint64_t* rbar = tempty + 2;  // per epilogue warp: its residual / history-base blocks landed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rbar + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -137,10 +143,13 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(&tfull[a], 1);
       mbar_init(&tempty[a], 256);
     }
+    for (int w = 0; w < 8; ++w) mbar_init(&rbar[w], 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
+    if (tm.pre & 1) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmR) : "memory");
+    if (tm.pre & 2) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmHB) : "memory");
     if (tm.n_tiles > tm.n_norm) {
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmW128) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA256) : "memory");
@@ -255,11 +264,11 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
           const bool in = m < M && n0 + 8 * k < N;
-          if (e.resid)
+          if (e.resid && !(tm.pre & 1))
             pr[k] = in ? *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.resid) +
                                                           (size_t)m * e.ld_resid + n0 + 8 * k)
                        : make_uint4(0, 0, 0, 0);
-          if (e.hist_out)
+          if (e.hist_out && !(tm.pre & 2))
             ph[k] = in ? *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.hist_base) +
                                                           (size_t)m * e.ldo + n0 + 8 * k)
                        : make_uint4(0, 0, 0, 0);
@@ -271,6 +280,30 @@ __global__ void __launch_bounds__(THREADS, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
+      // One tile per CTA: the ring's last readers (this tile's MMAs) are
+      // complete, so the warp's residual / history-base blocks (4 x 32 x 32
+      // bf16 each, 64-byte swizzle: the layout of the output blocks) come by
+      // TMA into its 8 KB slices of the ring; waited for at first use.
+      uint8_t* rsm = smem + (warp - 2) * 8192;
+      uint8_t* hsm = smem + 65536 + (warp - 2) * 8192;
+      bool pre_wait = tm.pre != 0;
+      if (tm.pre && lane == 0) {
+        mbar_expect_tx(&rbar[warp - 2], ((tm.pre & 1) ? 8192u : 0u) + ((tm.pre & 2) ? 8192u : 0u));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int x = t.sw ? t.n0 + q * 32 : t.n0 + c_lo + 32 * i;
+          const int y = t.sw ? t.m0 + h * (BN / 2) + 32 * i : t.m0 + q * 32;
+          if (tm.pre & 1) tma_load(&tmR, &rbar[warp - 2], rsm + i * 2048, x, y);
+          if (tm.pre & 2) tma_load(&tmHB, &rbar[warp - 2], hsm + i * 2048, x, y);
+        }
+      }
+      auto pre_ready = [&]() -> bool {
+        if (!pre_wait) return true;
+        pre_wait = false;
+        int w = 1;
+        if (lane == 0) w = mbar_wait_g(&rbar[warp - 2], 0, abort_flag) ? 1 : 0;
+        return __shfl_sync(0xffffffffu, w, 0) != 0;
+      };
       const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
       if (!t.sw && (C::XPOSE_BYTES == 0 || !tm.staged)) {
         const int m = t.m0 + row;
@@ -307,6 +340,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             for (int j = 0; j < 32; ++j) {
               const float g0 = __shfl_sync(0xffffffffu, pg0, j), g1 = __shfl_sync(0xffffffffu, pg1, j);
               v[j] *= lo ? g0 : g1;
+            }
+          }
+          if (tm.pre) {
+            if (!pre_ready()) { ok = 0; break; }
+            const uint8_t* rb = rsm + ((c - c_lo) >> 5) * 2048;
+            const uint8_t* hb2 = hsm + ((c - c_lo) >> 5) * 2048;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              if (tm.pre & 1) pr[k] = *reinterpret_cast<const uint4*>(rb + blk_off(lane, k));
+              if (tm.pre & 2) ph[k] = *reinterpret_cast<const uint4*>(hb2 + blk_off(lane, k));
             }
           }
           uint32_t ob[16], hb[16];
@@ -376,9 +419,61 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
           for (int j = 0; j < 16; ++j) v[j] = xp[r * 32 + ((c0 + j) ^ r)];  // out[m0 + r][n + c0 + j]
           __syncwarp();
-          if (m0 + r < M) epi_chunk<bf16, 16>(e, m0 + r, n + c0, N, v);
+          const int m = m0 + r;
+          if (tm.pre && !e.out_f32 && e.split_col >= N) {
+            // residual / history base of row m from the warp's ring slices
+            // (block (row in the warp's 128 rows) / 32, 16-byte chunks
+            // c0 / 8 and c0 / 8 + 1 of that row)
+            if (!pre_ready()) break;
+            if (m < M) {
+              epi_math<bf16, 16>(e, m, n + c0, N, v);
+              const int rw = c - h * (BN / 2) + r;
+              const uint32_t base = (uint32_t)((rw >> 5) * 2048);
+#pragma unroll
+              for (int g = 0; g < 2; ++g) {
+                const int nc = n + c0 + 8 * g;
+                if (nc >= N) continue;
+                const uint32_t off = base + blk_off(rw & 31, (c0 >> 3) + g);
+                uint4 rv = make_uint4(0, 0, 0, 0), hv = make_uint4(0, 0, 0, 0);
+                if (tm.pre & 1)
+                  rv = *reinterpret_cast<const uint4*>(rsm + off);
+                else if (e.resid)
+                  rv = *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.resid) + (size_t)m * e.ld_resid + nc);
+                if (e.hist_out)
+                  hv = (tm.pre & 2) ? *reinterpret_cast<const uint4*>(hsm + off)
+                                    : *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.hist_base) +
+                                                                      (size_t)m * e.ldo + nc);
+                const uint32_t rr4[4] = {rv.x, rv.y, rv.z, rv.w}, hh4[4] = {hv.x, hv.y, hv.z, hv.w};
+                uint32_t ob[4], hb[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  float a = v[8 * g + 2 * i], b = v[8 * g + 2 * i + 1];
+                  if (e.resid) {
+                    const float2 r2 = unpack2(rr4[i]);
+                    a += r2.x;
+                    b += r2.y;
+                  }
+                  ob[i] = pack2(a, b);
+                  if (e.hist_out) {  // stored(out) - hist_base
+                    const float2 o2 = unpack2(ob[i]), h2 = unpack2(hh4[i]);
+                    hb[i] = pack2(o2.x - h2.x, o2.y - h2.y);
+                  }
+                }
+                *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(e.out) + (size_t)m * e.ldo + nc) =
+                    make_uint4(ob[0], ob[1], ob[2], ob[3]);
+                if (e.hist_out)
+                  *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(e.hist_out) + (size_t)m * e.ldo + nc) =
+                      make_uint4(hb[0], hb[1], hb[2], hb[3]);
+              }
+            }
+            continue;
+          }
+          if (m < M) epi_chunk<bf16, 16>(e, m, n + c0, N, v);
         }
       }
+      // a warp whose columns all lie past N never read its blocks: their
+      // copies still land before it moves on
+      if (pre_wait) pre_ready();
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
     }
@@ -675,8 +770,9 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
   const long long t256 = (long long)tm.num_m * (N / 256) + (rem ? (long long)((rem + 127) / 128) * tm.num_m2 : 0);
   const long long t128 = (long long)tm.num_m * ((N + 127) / 128);
   const bool wide = (t256 + g_sms - 1) / g_sms <= (t128 + g_sms - 1) / g_sms;
-  CUtensorMap mw128 = {}, ma256 = {}, mo = {}, mh = {};
+  CUtensorMap mw128 = {}, ma256 = {}, mo = {}, mh = {}, mr = {}, mhb = {};
   tm.staged = 0;
+  tm.pre = 0;
   if (wide) {
     tm.n_full = N / 256;
     tm.n_norm = tm.num_m * tm.n_full;
@@ -693,15 +789,22 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
     if (!e.out_f32 && e.split_col >= N && aligned && gate_ok && make_store_map(&mo, e.out, M, N, e.ldo) &&
         (!e.hist_out || make_store_map(&mh, e.hist_out, M, N, e.ldo)))
       tm.staged = 1;
+    // one tile per CTA: residual / history-base blocks by TMA into the idle
+    // ring (16-byte aligned rows; otherwise the per-lane loads stay)
+    if (tm.staged && t256 <= g_sms) {
+      if (e.resid && make_store_map(&mr, const_cast<void*>(e.resid), M, N, e.ld_resid)) tm.pre |= 1;
+      if (e.hist_out && make_store_map(&mhb, const_cast<void*>(e.hist_base), M, N, e.ldo)) tm.pre |= 2;
+    }
     const int grid = (int)(t256 < g_sms ? t256 : g_sms);
-    launch_pdl(k_gemm_tc<256>, grid, THREADS, Cfg<256>::SMEM, s, ma, mb, mw128, ma256, mo, mh, M, N, K, tm, e);
+    launch_pdl(k_gemm_tc<256>, grid, THREADS, Cfg<256>::SMEM, s, ma, mb, mw128, ma256, mo, mh, mr, mhb, M, N, K, tm,
+               e);
   } else {
     tm.n_full = (N + 127) / 128;
     tm.n_norm = tm.num_m * tm.n_full;
     tm.n_tiles = tm.n_norm;
     if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, 128)) return cudaErrorInvalidValue;
     const int grid = (int)(t128 < g_sms ? t128 : g_sms);
-    launch_pdl(k_gemm_tc<128>, grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, M, N, K, tm, e);
+    launch_pdl(k_gemm_tc<128>, grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, ma, mb, M, N, K, tm, e);
   }
   return launched();
 }
