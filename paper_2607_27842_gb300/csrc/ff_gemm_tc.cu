@@ -4,18 +4,23 @@
 // Persistent kernel, one CTA per SM, 10 warps:
 //   warp 0      TMA producer: A and W tiles (128 and BN rows x 64 k, 128-byte
 //               swizzle) into a STAGES-deep shared-memory ring;
-//   warp 1      TMEM allocator and the single MMA-issuing thread:
+//   warp 1      TMEM allocator and MMA issuer (the whole warp runs the loop,
+//               one elected lane issues):
 //               tcgen05.mma.cta_group::1.kind::f16 (M = 128, N = BN, K = 16),
 //               fp32 accumulators in TMEM, tcgen05.commit frees ring slots;
 //   warps 2..9  epilogue: tcgen05.ld of the accumulator (each warp one
 //               32-lane quarter and one column half), the fused bias / RoPE /
-//               GELU / gate / residual / history epilogue, 16-byte stores.
+//               GELU / gate / residual / history epilogue, stores through
+//               swizzled shared-memory blocks and TMA (16-byte stores where
+//               the output does not allow it); with one tile per CTA the
+//               residual / history-base blocks arrive by TMA as well.
 // Two TMEM accumulators (2 * BN columns) let the epilogue of tile i overlap
 // the main loop of tile i + 1.  Every mbarrier wait is bounded: on timeout
 // the CTA raises a watchdog flag, stops issuing work and releases its TMEM.
 //
-// A 128 x 128 x 16 MMA takes about as long as a 128 x 256 x 16 one, so
-// narrow tiles run at half rate.  With BN = 256 the columns past the last
+// With both operands in shared memory a 128 x 128 x 16 MMA is bound by the
+// operand reads and takes about as long as a 128 x 256 x 16 one, so narrow
+// tiles run at half rate.  With BN = 256 the columns past the last
 // full 256-wide tile are covered by swapped tiles: up to 128 rows of W as
 // the MMA's M side against 256 rows of A as its N side (the accumulator
 // holds the transposed block; the epilogue transposes it back through a
