@@ -126,6 +126,23 @@ __device__ __forceinline__ void tmem_ld64w(uint32_t taddr, float* v) {
       : "r"(taddr)
       : "memory");
 }
+// 32 TMEM columns without waiting; tmem_wait32 on the same registers
+// completes them (its in/out operands keep every use behind the wait)
+__device__ __forceinline__ void tmem_ld32_async(uint32_t taddr, float* v) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n"
+               : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]), "=f"(v[7]), "=f"(v[8]), "=f"(v[9]), "=f"(v[10]), "=f"(v[11]), "=f"(v[12]), "=f"(v[13]), "=f"(v[14]), "=f"(v[15]), "=f"(v[16]), "=f"(v[17]), "=f"(v[18]), "=f"(v[19]), "=f"(v[20]), "=f"(v[21]), "=f"(v[22]), "=f"(v[23]), "=f"(v[24]), "=f"(v[25]), "=f"(v[26]), "=f"(v[27]), "=f"(v[28]), "=f"(v[29]), "=f"(v[30]), "=f"(v[31])
+               : "r"(taddr)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_wait32(float* v) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;\n" : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]), "+f"(v[6]), "+f"(v[7]), "+f"(v[8]), "+f"(v[9]), "+f"(v[10]), "+f"(v[11]), "+f"(v[12]), "+f"(v[13]), "+f"(v[14]), "+f"(v[15]), "+f"(v[16]), "+f"(v[17]), "+f"(v[18]), "+f"(v[19]), "+f"(v[20]), "+f"(v[21]), "+f"(v[22]), "+f"(v[23]), "+f"(v[24]), "+f"(v[25]), "+f"(v[26]), "+f"(v[27]), "+f"(v[28]), "+f"(v[29]), "+f"(v[30]), "+f"(v[31]) : : "memory");
+}
+__device__ __forceinline__ void tmem_st16u(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};\n" ::"r"(taddr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+               "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+               : "memory");
+}
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};\n" ::"r"(taddr),
@@ -337,21 +354,41 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       if (lane == 0) w = wait_a(&s_full[i], j & 1, abort_flag) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
       tc_fence_after();
-      float v[AKV];
-      tmem_ld64w(s_col, v);
-      tmem_ld64w(s_col + 64, v + 64);
-      if (valid < AKV) {
-#pragma unroll
-        for (int e = 0; e < AKV; ++e)
-          if (e >= valid) v[e] = -INFINITY;
-      }
       // row max as a tree of three-input maxima (72 instructions for 128
-      // values instead of 127)
+      // values instead of 127).  One query tile per CTA (short sequences,
+      // latency-bound): S is read 64 columns at a time for the max and again
+      // in quarters for the exponentials, which keeps the row out of
+      // registers; two query tiles: the row is held in registers.
+      float v[QT == 1 ? 1 : AKV];
       float mx[16];
+      if constexpr (QT == 1) {
 #pragma unroll
-      for (int e = 0; e < 16; ++e)
-        mx[e] = max3f(max3f(v[e], v[e + 16], v[e + 32]), max3f(v[e + 48], v[e + 64], v[e + 80]),
-                      fmaxf(v[e + 96], v[e + 112]));
+        for (int e = 0; e < 16; ++e) mx[e] = -INFINITY;
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          float t[64];
+          tmem_ld64w(s_col + (uint32_t)(64 * hh), t);
+          if (valid < AKV) {
+#pragma unroll
+            for (int e = 0; e < 64; ++e)
+              if (64 * hh + e >= valid) t[e] = -INFINITY;
+          }
+#pragma unroll
+          for (int e = 0; e < 16; ++e) mx[e] = max3f(mx[e], max3f(t[e], t[e + 16], t[e + 32]), t[e + 48]);
+        }
+      } else {
+        tmem_ld64w(s_col, v);
+        tmem_ld64w(s_col + 64, v + 64);
+        if (valid < AKV) {
+#pragma unroll
+          for (int e = 0; e < AKV; ++e)
+            if (e >= valid) v[e] = -INFINITY;
+        }
+#pragma unroll
+        for (int e = 0; e < 16; ++e)
+          mx[e] = max3f(max3f(v[e], v[e + 16], v[e + 32]), max3f(v[e + 48], v[e + 64], v[e + 80]),
+                        fmaxf(v[e + 96], v[e + 112]));
+      }
 #pragma unroll
       for (int e = 0; e < 5; ++e) mx[e] = max3f(mx[e], mx[e + 5], mx[e + 10]);
       mx[0] = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[15]), mx[0]);
@@ -376,18 +413,48 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
 #pragma unroll
       for (int e = 0; e < 8; ++e) ls[e] = 0.f;
       // P as bf16 pairs into the first 64 columns of S_i (already read)
+      if constexpr (QT == 1) {
+        // S again, 32 columns at a time (the next quarter loading while this
+        // one is finished); quarter k's P columns [16k, 16k + 16) lie in
+        // columns already read
+        float sq[2][32];
+        tmem_ld32_async(s_col, sq[0]);
+        tmem_wait32(sq[0]);
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        uint32_t pk[32];
+        for (int k = 0; k < 4; ++k) {
+          if (k + 1 < 4) tmem_ld32_async(s_col + (uint32_t)(32 * (k + 1)), sq[(k + 1) & 1]);
+          float* x = sq[k & 1];
+          if (valid < AKV) {
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const float p0 = ex2(fmaf(v[half * 64 + 2 * e], scale_log2, -m));
-          const float p1 = ex2(fmaf(v[half * 64 + 2 * e + 1], scale_log2, -m));
-          ls[e & 7] += p0 + p1;
-          __nv_bfloat162 t2 = __floats2bfloat162_rn(p0, p1);
-          pk[e] = *reinterpret_cast<uint32_t*>(&t2);
+            for (int e = 0; e < 32; ++e)
+              if (32 * k + e >= valid) x[e] = -INFINITY;
+          }
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const float p0 = ex2(fmaf(x[2 * e], scale_log2, -m));
+            const float p1 = ex2(fmaf(x[2 * e + 1], scale_log2, -m));
+            ls[e & 7] += p0 + p1;
+            __nv_bfloat162 t2 = __floats2bfloat162_rn(p0, p1);
+            pk[e] = *reinterpret_cast<uint32_t*>(&t2);
+          }
+          tmem_st16u(s_col + (uint32_t)(16 * k), pk);
+          if (k + 1 < 4) tmem_wait32(sq[(k + 1) & 1]);
         }
-        tmem_st32(s_col + (uint32_t)(half * 32), pk);
+      } else {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const float p0 = ex2(fmaf(v[half * 64 + 2 * e], scale_log2, -m));
+            const float p1 = ex2(fmaf(v[half * 64 + 2 * e + 1], scale_log2, -m));
+            ls[e & 7] += p0 + p1;
+            __nv_bfloat162 t2 = __floats2bfloat162_rn(p0, p1);
+            pk[e] = *reinterpret_cast<uint32_t*>(&t2);
+          }
+          tmem_st32(s_col + (uint32_t)(half * 32), pk);
+        }
       }
       l = l * alpha + (((ls[0] + ls[1]) + (ls[2] + ls[3])) + ((ls[4] + ls[5]) + (ls[6] + ls[7])));
       tmem_st_wait();
