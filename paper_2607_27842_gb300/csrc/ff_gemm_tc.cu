@@ -409,6 +409,22 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int n = t.n0 + q * 32;
         if (lane == 0) bulk_wait_read<0>();  // TMA stores of earlier tiles done reading the buffer
         __syncwarp();
+        // preloaded form: the lane's 16 columns are the same for every block
+        // of rows, so their bias stays in registers and the gate row is
+        // reloaded only when the row's sample changes
+        const bool pre_sw = tm.pre && !e.out_f32 && e.split_col >= N && !e.rope;
+        float bv[16], gv[16];
+        int gb = -1;
+        if (pre_sw) {
+          const int nc0 = n + (lane & 1) * 16;
+#pragma unroll
+          for (int g = 0; g < 2; ++g) {
+            float b8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            if (e.bias && nc0 + 8 * g < N) ld16(reinterpret_cast<const bf16*>(e.bias) + nc0 + 8 * g, b8);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) bv[8 * g + k] = b8[k];
+          }
+        }
         for (int c = h * (BN / 2); c < (h + 1) * (BN / 2) && n < N; c += 16) {
           const int m0 = t.m0 + c;
           if (m0 >= M) break;
@@ -431,7 +447,28 @@ __global__ void __launch_bounds__(THREADS, 1)
             // c0 / 8 and c0 / 8 + 1 of that row)
             if (!pre_ready()) break;
             if (m < M) {
-              epi_math<bf16, 16>(e, m, n + c0, N, v);
+              if (pre_sw) {  // epi_math's order: act(acc + bias) * gate
+#pragma unroll
+                for (int j = 0; j < 16; ++j) v[j] += bv[j];
+                epi_rope_act<bf16, 16>(e, m, n + c0, v);
+                if (e.gate) {
+                  const int bt = epi_batch(e, m);
+                  if (bt != gb) {
+                    gb = bt;
+                    const float* gp = e.gate + (size_t)bt * e.gate_stride + n + c0;
+#pragma unroll
+                    for (int j = 0; j < 16; j += 4) {
+                      const float4 g4 = n + c0 + j < N ? *reinterpret_cast<const float4*>(gp + j)
+                                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+                      gv[j] = g4.x; gv[j + 1] = g4.y; gv[j + 2] = g4.z; gv[j + 3] = g4.w;
+                    }
+                  }
+#pragma unroll
+                  for (int j = 0; j < 16; ++j) v[j] *= gv[j];
+                }
+              } else {
+                epi_math<bf16, 16>(e, m, n + c0, N, v);
+              }
               const int rw = c - h * (BN / 2) + r;
               const uint32_t base = (uint32_t)((rw >> 5) * 2048);
 #pragma unroll
