@@ -38,6 +38,7 @@
 #include <cudaTypedefs.h>
 
 #include <math.h>
+#include <algorithm>
 #include <mutex>
 
 namespace ff {
@@ -188,7 +189,7 @@ __device__ __forceinline__ SegTile seg_tile(const AttnArgs& a, int b, int t) {
 
 template <int D, int QT>
 __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
-    k_attn_tc(const __grid_constant__ CUtensorMap tmQKV, AttnArgs a, float scale_log2) {
+    k_attn_tc(const __grid_constant__ CUtensorMap tmQKV, AttnArgs a, float scale_log2, int ipc) {
   using C = ACfg<D, QT>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -204,12 +205,18 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
   uint64_t* s_full = v_empty + C::VST;       // per query tile
   uint64_t* p_ready = s_full + 2;            // per query tile
   uint64_t* o_final = p_ready + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_final + 1);
+  uint64_t* q_empty = o_final + 1;           // Q tiles free for the CTA's next item
+  uint64_t* o_free = q_empty + 1;            // O read out by the softmax warps' epilogue
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_free + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y, b = blockIdx.z;
-  const int nkv = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;
+  const int nkv = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;  // key tiles = query tiles of a sample
+  // item it of this CTA: query tiles QT * (blockIdx.x * ipc + it) + i; the
+  // key / value rings, s_full and p_ready count on across items (kv step
+  // jj = it * nkv + j)
+  auto item_live = [&](int it) { return QT * (blockIdx.x * ipc + it) < nkv; };
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
@@ -226,6 +233,8 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       mbar_init(&p_ready[i], 128);
     }
     mbar_init(o_final, 1);
+    mbar_init(q_empty, 1);
+    mbar_init(o_free, 128 * QT);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQKV) : "memory");
@@ -247,25 +256,32 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      mbar_expect_tx(q_full, QT * C::TILE);
-      for (int i = 0; i < QT; ++i) {
-        const SegTile qs = seg_tile(a, b, QT * blockIdx.x + i);
-        for (int bx = 0; bx < C::NBOX; ++bx) tma_load3(&tmQKV, q_full, sQ + i * C::TILE + bx * C::BOX, 64 * bx, h, qs.row0);
-      }
       int nk = 0, nv = 0;
-      for (int j = 0; j < nkv; ++j) {
-        const SegTile ks = seg_tile(a, b, j);
-        const int sk = j % C::KST, sv = j % C::VST;
-        if (!wait_a(&k_empty[sk], ((j / C::KST) & 1) ^ 1, abort_flag)) break;
-        mbar_expect_tx(&k_full[sk], C::TILE);
-        for (int bx = 0; bx < C::NBOX; ++bx)
-          tma_load3(&tmQKV, &k_full[sk], sK + sk * C::TILE + bx * C::BOX, 64 * bx, a.H + h, ks.row0);
-        ++nk;
-        if (!wait_a(&v_empty[sv], ((j / C::VST) & 1) ^ 1, abort_flag)) break;
-        mbar_expect_tx(&v_full[sv], C::TILE);
-        for (int bx = 0; bx < C::NBOX; ++bx)
-          tma_load3(&tmQKV, &v_full[sv], sV + sv * C::TILE + bx * C::BOX, 64 * bx, 2 * a.H + h, ks.row0);
-        ++nv;
+      bool ok = true;
+      for (int it = 0; it < ipc && ok && item_live(it); ++it) {
+        // the next item's Q waits for the previous item's last S MMAs
+        if (it > 0 && !wait_a(q_empty, (it - 1) & 1, abort_flag)) break;
+        mbar_expect_tx(q_full, QT * C::TILE);
+        for (int i = 0; i < QT; ++i) {
+          const SegTile qs = seg_tile(a, b, QT * (blockIdx.x * ipc + it) + i);
+          for (int bx = 0; bx < C::NBOX; ++bx)
+            tma_load3(&tmQKV, q_full, sQ + i * C::TILE + bx * C::BOX, 64 * bx, h, qs.row0);
+        }
+        for (int j = 0; j < nkv; ++j) {
+          const int jj = it * nkv + j;
+          const SegTile ks = seg_tile(a, b, j);
+          const int sk = jj % C::KST, sv = jj % C::VST;
+          if (!wait_a(&k_empty[sk], ((jj / C::KST) & 1) ^ 1, abort_flag)) { ok = false; break; }
+          mbar_expect_tx(&k_full[sk], C::TILE);
+          for (int bx = 0; bx < C::NBOX; ++bx)
+            tma_load3(&tmQKV, &k_full[sk], sK + sk * C::TILE + bx * C::BOX, 64 * bx, a.H + h, ks.row0);
+          ++nk;
+          if (!wait_a(&v_empty[sv], ((jj / C::VST) & 1) ^ 1, abort_flag)) { ok = false; break; }
+          mbar_expect_tx(&v_full[sv], C::TILE);
+          for (int bx = 0; bx < C::NBOX; ++bx)
+            tma_load3(&tmQKV, &v_full[sv], sV + sv * C::TILE + bx * C::BOX, 64 * bx, 2 * a.H + h, ks.row0);
+          ++nv;
+        }
       }
       // Copies still in flight complete on their full barriers; wait for the
       // last ring's worth of each so none lands after the CTA exits.
@@ -283,12 +299,12 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       }
     }
   } else if (warp == 1) {
-    bool ok = wait_u(q_full, 0, abort_flag);
+    bool ok = true;
     const uint64_t qd0 = sw128_desc(saddr(sQ)), qd1 = sw128_desc(saddr(sQ + C::TILE));
-    // S_i = Q_i K_j^T (DK / 16 steps of 16 along the head width: box k / 4,
+    // S_i = Q_i K_jj^T (DK / 16 steps of 16 along the head width: box k / 4,
     // +32 B per step inside the box), then arrive on s_full[i]
-    auto issue_s = [&](int i, int j) {
-      const uint64_t kd = sw128_desc(saddr(sK + (j % C::KST) * C::TILE));
+    auto issue_s = [&](int i, int jj) {
+      const uint64_t kd = sw128_desc(saddr(sK + (jj % C::KST) * C::TILE));
       const uint64_t qd = i ? qd1 : qd0;
 #pragma unroll
       for (int k = 0; k < C::DK / 16; ++k) {
@@ -297,46 +313,56 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       }
       if (elect_one()) umma_commit(&s_full[i]);
     };
-    if (ok) ok = wait_u(&k_full[0], 0, abort_flag);
-    if (ok) {
+    for (int it = 0; it < ipc && ok && item_live(it); ++it) {
+      const int jb = it * nkv;  // the item's first kv step
+      ok = wait_u(q_full, it & 1, abort_flag);
+      if (ok) ok = wait_u(&k_full[jb % C::KST], (jb / C::KST) & 1, abort_flag);
+      if (!ok) break;
       tc_fence_after();
-      issue_s(0, 0);
-      if (QT == 2) issue_s(1, 0);
-      if (elect_one()) umma_commit(&k_empty[0]);
-      ok = wait_u(&v_full[0], 0, abort_flag);
-    }
-    // Per key tile j: [p_ready 0] O_0 += P_0 V_j [k_full j+1] S_0 for j + 1
-    // [p_ready 1] O_1 += P_1 V_j [v_full j+1] S_1 for j + 1 -- one wait in
-    // each gap between MMA groups
-    for (int j = 0; j < nkv && ok; ++j) {
-      const int sv = j % C::VST;
-      const bool more = j + 1 < nkv;
-      const uint32_t vaddr = saddr(sV + sv * C::TILE);
-      for (int i = 0; i < QT; ++i) {
-        ok = wait_u(&p_ready[i], j & 1, abort_flag);
-        if (!ok) break;
-        tc_fence_after();
-        // O_i += P_i V_j: 16 keys per step = 8 TMEM columns of P, 2 groups
-        // of 8 value rows (2 KB) of the MN-major V tile
-#pragma unroll
-        for (int k = 0; k < AKV / 16; ++k) {
-          const uint64_t vd = sw128_desc_mn(vaddr + (uint32_t)k * 2048u, C::BOX);
-          if (elect_one())
-            umma_ts(tmem + C::TMEM_O + (uint32_t)(i * AKV), tmem + (uint32_t)(i * AKV + k * 8), vd, C::IDESC_O,
-                    (j | k) != 0);
-        }
-        if (i == QT - 1 && elect_one()) umma_commit(&v_empty[sv]);
-        if (more) {
-          if (i == 0) ok = wait_u(&k_full[(j + 1) % C::KST], ((j + 1) / C::KST) & 1, abort_flag);
-          if (ok && i == QT - 1) ok = wait_u(&v_full[(j + 1) % C::VST], ((j + 1) / C::VST) & 1, abort_flag);
+      issue_s(0, jb);
+      if (QT == 2) issue_s(1, jb);
+      if (elect_one()) umma_commit(&k_empty[jb % C::KST]);
+      if (nkv == 1 && elect_one()) umma_commit(q_empty);  // the item's last S MMAs
+      ok = wait_u(&v_full[jb % C::VST], (jb / C::VST) & 1, abort_flag);
+      // the previous item's O has been read out before this item's first P V
+      if (ok && it > 0) ok = wait_u(o_free, (it - 1) & 1, abort_flag);
+      // Per key tile j: [p_ready 0] O_0 += P_0 V_j [k_full j+1] S_0 for j + 1
+      // [p_ready 1] O_1 += P_1 V_j [v_full j+1] S_1 for j + 1 -- one wait in
+      // each gap between MMA groups
+      for (int j = 0; j < nkv && ok; ++j) {
+        const int jj = jb + j;
+        const int sv = jj % C::VST;
+        const bool more = j + 1 < nkv;
+        const uint32_t vaddr = saddr(sV + sv * C::TILE);
+        for (int i = 0; i < QT; ++i) {
+          ok = wait_u(&p_ready[i], jj & 1, abort_flag);
           if (!ok) break;
           tc_fence_after();
-          issue_s(i, j + 1);  // behind O_i's update: the MMA pipe reads P_i before S_i is overwritten
-          if (i == QT - 1 && elect_one()) umma_commit(&k_empty[(j + 1) % C::KST]);
+          // O_i += P_i V_j: 16 keys per step = 8 TMEM columns of P, 2 groups
+          // of 8 value rows (2 KB) of the MN-major V tile
+#pragma unroll
+          for (int k = 0; k < AKV / 16; ++k) {
+            const uint64_t vd = sw128_desc_mn(vaddr + (uint32_t)k * 2048u, C::BOX);
+            if (elect_one())
+              umma_ts(tmem + C::TMEM_O + (uint32_t)(i * AKV), tmem + (uint32_t)(i * AKV + k * 8), vd, C::IDESC_O,
+                      (j | k) != 0);
+          }
+          if (i == QT - 1 && elect_one()) umma_commit(&v_empty[sv]);
+          if (more) {
+            if (i == 0) ok = wait_u(&k_full[(jj + 1) % C::KST], ((jj + 1) / C::KST) & 1, abort_flag);
+            if (ok && i == QT - 1) ok = wait_u(&v_full[(jj + 1) % C::VST], ((jj + 1) / C::VST) & 1, abort_flag);
+            if (!ok) break;
+            tc_fence_after();
+            issue_s(i, jj + 1);  // behind O_i's update: the MMA pipe reads P_i before S_i is overwritten
+            if (i == QT - 1 && elect_one()) {
+              umma_commit(&k_empty[(jj + 1) % C::KST]);
+              if (j + 2 == nkv) umma_commit(q_empty);  // the item's last S MMAs
+            }
+          }
         }
       }
+      if (ok && elect_one()) umma_commit(o_final);
     }
-    if (ok && elect_one()) umma_commit(o_final);
   } else if (warp >= C::SOFT_WARP0) {
     // softmax of query tile i: row r of the tile = TMEM lane r
     const int i = (warp - C::SOFT_WARP0) >> 2;
@@ -345,13 +371,14 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const uint32_t s_col = tmem + lane_off + (uint32_t)(i * AKV);
     const uint32_t o_col = tmem + lane_off + C::TMEM_O + (uint32_t)(i * AKV);
-    const SegTile qs = seg_tile(a, b, QT * blockIdx.x + i);
-    float m = -INFINITY, l = 0.f;
     bool ok = true;
+    for (int it = 0; it < ipc && ok && item_live(it); ++it) {
+    const SegTile qs = seg_tile(a, b, QT * (blockIdx.x * ipc + it) + i);
+    float m = -INFINITY, l = 0.f;
     for (int j = 0; j < nkv; ++j) {
       const int valid = seg_tile(a, b, j).valid;
       int w = 1;
-      if (lane == 0) w = wait_a(&s_full[i], j & 1, abort_flag) ? 1 : 0;
+      if (lane == 0) w = wait_a(&s_full[i], (it * nkv + j) & 1, abort_flag) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
       tc_fence_after();
       // row max as a tree of three-input maxima (72 instructions for 128
@@ -461,30 +488,32 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       tc_fence_before();
       mbar_arrive(&p_ready[i]);
     }
-    if (ok) {
-      int w = 1;
-      if (lane == 0) w = wait_a(o_final, 0, abort_flag) ? 1 : 0;
-      if (__shfl_sync(0xffffffffu, w, 0)) {
-        tc_fence_after();
-        const float inv = 1.0f / l;
-        bf16* orow = reinterpret_cast<bf16*>(a.out) + (size_t)(qs.row0 + (r < qs.valid ? r : 0)) * a.ld_out + (size_t)h * D;
+    if (!ok) break;
+    int w = 1;
+    if (lane == 0) w = wait_a(o_final, it & 1, abort_flag) ? 1 : 0;
+    if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+    tc_fence_after();
+    const float inv = 1.0f / l;
+    bf16* orow = reinterpret_cast<bf16*>(a.out) + (size_t)(qs.row0 + (r < qs.valid ? r : 0)) * a.ld_out + (size_t)h * D;
 #pragma unroll
-        for (int c = 0; c < C::DK / 16; ++c) {
-          float o[16];
-          tmem_ld16(o_col + (uint32_t)(c * 16), o);
-          if (r < qs.valid) {
+    for (int c = 0; c < C::DK / 16; ++c) {
+      float o[16];
+      tmem_ld16(o_col + (uint32_t)(c * 16), o);
+      if (r < qs.valid) {
 #pragma unroll
-            for (int e = 0; e < 16; e += 8) {
-              if (c * 16 + e < D) {
-                float t8[8];
+        for (int e = 0; e < 16; e += 8) {
+          if (c * 16 + e < D) {
+            float t8[8];
 #pragma unroll
-                for (int z = 0; z < 8; ++z) t8[z] = o[e + z] * inv;
-                st16(orow + c * 16 + e, t8);
-              }
-            }
+            for (int z = 0; z < 8; ++z) t8[z] = o[e + z] * inv;
+            st16(orow + c * 16 + e, t8);
           }
         }
       }
+    }
+    // O is read out: the next item's first P V may overwrite it
+    tc_fence_before();
+    mbar_arrive(o_free);
     }
   }
   tc_fence_before();
@@ -498,6 +527,7 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
 
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
 std::once_flag g_once;
+int g_attn_sms = 148;
 
 bool init_attn() {
   std::call_once(g_once, [] {
@@ -506,6 +536,10 @@ bool init_attn() {
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
         q == cudaDriverEntryPointSuccess)
       g_enc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
+        sms > 0)
+      g_attn_sms = sms;
 #define FF_ATTR(d, qt) \
   cudaFuncSetAttribute(k_attn_tc<d, qt>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ACfg<d, qt>::SMEM)
     FF_ATTR(64, 1); FF_ATTR(64, 2); FF_ATTR(72, 1); FF_ATTR(72, 2); FF_ATTR(128, 1); FF_ATTR(128, 2);
@@ -534,10 +568,16 @@ cudaError_t attn_tc_t(const AttnArgs& a, cudaStream_t s) {
   const int nq = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)D);
   if (nq <= SHORT_KV_TILES) {
-    launch_pdl(k_attn_tc<D, 1>, dim3(nq, a.H, a.B), ACfg<D, 1>::THREADS, ACfg<D, 1>::SMEM, s, tm, a, scale_log2);
+    // query tiles of one (sample, head) per CTA: as few as keep the CTAs
+    // within one wave of two per SM, so the second tile's loads overlap the
+    // first tile's tail instead of a second wave starting from scratch
+    const long long items = (long long)nq * a.H * a.B, slots = 2LL * g_attn_sms;
+    const int ipc = (int)std::min<long long>(nq, std::max<long long>(1, (items + slots - 1) / slots));
+    launch_pdl(k_attn_tc<D, 1>, dim3((nq + ipc - 1) / ipc, a.H, a.B), ACfg<D, 1>::THREADS, ACfg<D, 1>::SMEM, s, tm, a,
+               scale_log2, ipc);
   } else {
     launch_pdl(k_attn_tc<D, 2>, dim3((nq + 1) / 2, a.H, a.B), ACfg<D, 2>::THREADS, ACfg<D, 2>::SMEM, s, tm, a,
-               scale_log2);
+               scale_log2, 1);
   }
   return launched();
 }
