@@ -2,8 +2,8 @@
 // on the 5th-generation tensor cores, bf16 in, fp32 accumulate.
 //
 // One CTA per (sample, head, pair of 128-query tiles), 10 warps (sequences
-// of at most four key tiles: one query tile per CTA, 6 warps, two CTAs per
-// SM):
+// of at most four key tiles: 6 warps, two CTAs per SM, each CTA taking one
+// or more query tiles of its (sample, head) in turn):
 //   warp 0     TMA producer: both query tiles once, then key and value tiles
 //              of 128 tokens into separate rings, straight from the fused qkv
 //              activation (3-D tensor map: head width, head slot, row; the
@@ -71,7 +71,9 @@ __device__ __forceinline__ bool wait_u(uint64_t* b, uint32_t parity, volatile in
 // each other's MMAs, key / value rings as deep as shared memory allows, one
 // CTA per SM.  QT = 1 (short sequences, a couple of key tiles): one softmax
 // warpgroup, single-slot rings and half the TMEM, so two CTAs share an SM
-// and overlap their latency chains instead.
+// and overlap their latency chains instead; a CTA takes several query tiles
+// in turn so that all CTAs fit in one wave and a tile's loads overlap the
+// previous tile's tail.
 template <int D, int QT> struct ACfg {
   static constexpr int SOFT_WARP0 = 2;                   // first softmax warp
   static constexpr int THREADS = 32 * SOFT_WARP0 + 128 * QT;  // TMA warp, MMA warp, softmax warpgroups
