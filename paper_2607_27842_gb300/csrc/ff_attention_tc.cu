@@ -38,7 +38,6 @@
 #include <cudaTypedefs.h>
 
 #include <math.h>
-#include <algorithm>
 #include <mutex>
 
 namespace ff {
@@ -573,8 +572,9 @@ cudaError_t attn_tc_t(const AttnArgs& a, cudaStream_t s) {
     // query tiles of one (sample, head) per CTA: as few as keep the CTAs
     // within one wave of two per SM, so the second tile's loads overlap the
     // first tile's tail instead of a second wave starting from scratch
-    const long long items = (long long)nq * a.H * a.B, slots = 2LL * g_attn_sms;
-    const int ipc = (int)std::min<long long>(nq, std::max<long long>(1, (items + slots - 1) / slots));
+    const long long heads = (long long)a.H * a.B, slots = 2LL * g_attn_sms;
+    int ipc = 1;
+    while (ipc < nq && (long long)((nq + ipc - 1) / ipc) * heads > slots) ++ipc;
     launch_pdl(k_attn_tc<D, 1>, dim3((nq + ipc - 1) / ipc, a.H, a.B), ACfg<D, 1>::THREADS, ACfg<D, 1>::SMEM, s, tm, a,
                scale_log2, ipc);
   } else {
