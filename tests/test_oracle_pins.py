@@ -598,3 +598,157 @@ def test_flop_counter_matches_table_1():
     per_step = flops.step_flops(synthetic.SHAPES["flux"])
     assert per_step / 1e12 == pytest.approx(74.36, abs=0.01)
     assert abs(per_step / 1e12 / (3734.6 / 50) - 1) < 0.005
+
+
+# ----------------------------------------------------------------------------
+# conditioning, token embedding, output head and the sampler's use of the
+# head (Eq. 1's conditioning c, Section 3.1's samplers)
+# ----------------------------------------------------------------------------
+
+def torch_cond(W, t, labels, batch):
+    """c = Linear(SiLU(Linear(sinusoid(t)))) + label row, written with
+    torch.nn.functional and torch's own sinusoid."""
+    half = 128
+    freqs = torch.exp(-math.log(10000.0) * torch.arange(half, dtype=torch.float64) / half)
+    s = torch.cat([torch.cos(t * freqs), torch.sin(t * freqs)])
+    T = {k: t64(v) for k, v in W.items()}
+    e = F.linear(F.silu(F.linear(s, T["t_fc1.w"], T["t_fc1.b"])), T["t_fc2.w"], T["t_fc2.b"])
+    c = e[None].expand(batch, -1)
+    if labels is not None:
+        c = c + F.embedding(torch.as_tensor(labels), T["y_emb"])
+    return c.numpy()
+
+
+def test_cond_vector_matches_torch_composition():
+    sh = small_dit()
+    W = weights64(sh, seed=3, scale=20.0)       # large enough that SiLU is far from linear
+    labels = np.array([1, 4, 5, 5])              # the guidance half uses the null class 5
+    np.testing.assert_allclose(model.cond_vector(W, 437.0, labels=labels, batch=4),
+                               torch_cond(W, 437.0, labels, 4), rtol=1e-12, atol=1e-12)
+    Wm = weights64(small_mmdit(), seed=3, scale=20.0)
+    np.testing.assert_allclose(model.cond_vector(Wm, 12.5, batch=2), torch_cond(Wm, 12.5, None, 2),
+                               rtol=1e-12, atol=1e-12)
+
+
+def test_cond_vector_label_and_time_parts_separate():
+    """A zero label table leaves the time MLP alone, identical for every
+    sample; a zero time MLP output leaves exactly the label rows (so the
+    labels are added after the MLP, never fed through it)."""
+    sh = small_dit()
+    W = weights64(sh, seed=5, scale=10.0)
+    labels = np.array([0, 3, 5, 2])
+    Wy0 = dict(W, y_emb=np.zeros_like(W["y_emb"]))
+    c = model.cond_vector(Wy0, 250.0, labels=labels, batch=4)
+    h = model.silu(model.timestep_sinusoid(250.0) @ W["t_fc1.w"].T + W["t_fc1.b"])
+    np.testing.assert_allclose(c, np.tile(h @ W["t_fc2.w"].T + W["t_fc2.b"], (4, 1)), rtol=1e-12, atol=1e-13)
+    Wt0 = dict(W, **{"t_fc2.w": np.zeros_like(W["t_fc2.w"]), "t_fc2.b": np.zeros_like(W["t_fc2.b"])})
+    np.testing.assert_array_equal(model.cond_vector(Wt0, 250.0, labels=labels, batch=4), W["y_emb"][labels])
+
+
+def test_embed_tokens_dit_unit_impulse():
+    """One latent element set to 1: only its patch token moves, by the
+    column of the patch-embedding weight its (channel, row, column) offset
+    selects; every token carries bias + its 2-D sin-cos position."""
+    sh = small_dit(lat_h=8, lat_w=6)
+    W = weights64(sh, seed=7)
+    x = np.zeros((4, sh.in_ch, 8, 6))
+    x[1, 2, 5, 3] = 1.0
+    tok = model.embed_tokens(W, sh, x)
+    gw = 6 // 2
+    n_hot = (5 // 2) * gw + 3 // 2
+    f_hot = 2 * 4 + (5 % 2) * 2 + (3 % 2)
+    base = W["x_emb.b"][None, None] + model.sincos_pos_2d(sh.hidden, 4, gw)[None]
+    want = np.broadcast_to(base, tok.shape).copy()
+    want[1, n_hot] += W["x_emb.w"][:, f_hot]
+    np.testing.assert_allclose(tok, want, rtol=1e-13, atol=1e-13)
+
+
+def test_embed_tokens_mmdit_text_first_no_position():
+    """MMDiT: the text tokens come first, unchanged; the image tokens are
+    the patch embedding alone (positions enter through the rotary
+    embedding inside the blocks, not here)."""
+    sh = small_mmdit(lat_f=2, lat_h=4, lat_w=6, patch_t=1, rope_dims=3, head_dim=16)
+    W = weights64(sh, seed=9)
+    x = np.zeros((1, sh.in_ch, 2, 4, 6))
+    x[0, 3, 1, 2, 5] = 1.0
+    txt = rnd(1, sh.txt_tokens, sh.hidden)
+    tok = model.embed_tokens(W, sh, x, txt=txt)
+    assert tok.shape == (1, sh.txt_tokens + 2 * 2 * 3, sh.hidden)
+    np.testing.assert_array_equal(tok[:, :sh.txt_tokens], txt)
+    img = tok[:, sh.txt_tokens:]
+    n_hot = 1 * (2 * 3) + (2 // 2) * 3 + 5 // 2
+    f_hot = 3 * 4 + (2 % 2) * 2 + (5 % 2)
+    want = np.broadcast_to(W["img_in.b"], img.shape).copy()
+    want[0, n_hot] += W["img_in.w"][:, f_hot]
+    np.testing.assert_allclose(img, want, rtol=1e-13, atol=1e-13)
+
+
+def torch_final(W, sh, tok, c):
+    T = {k: t64(v) for k, v in W.items()}
+    img = t64(tok)[:, sh.txt_tokens:] if sh.arch == "mmdit" else t64(tok)
+    shift, scale = F.linear(F.silu(t64(c)), T["final.mod.w"], T["final.mod.b"]).chunk(2, dim=-1)
+    y = F.linear(F.layer_norm(img, (sh.hidden,), eps=1e-6) * (1 + scale[:, None]) + shift[:, None],
+                 T["final.lin.w"], T["final.lin.b"])
+    B, p = y.shape[0], sh.patch
+    gh, gw = sh.lat_h // p, sh.lat_w // p
+    if sh.lat_f > 0:
+        y = y.reshape(B, sh.lat_f, gh, gw, sh.out_ch, 1, p, p).permute(0, 4, 1, 5, 2, 6, 3, 7)
+        return y.reshape(B, sh.out_ch, sh.lat_f, sh.lat_h, sh.lat_w).numpy()
+    y = y.reshape(B, gh, gw, sh.out_ch, p, p).permute(0, 3, 1, 4, 2, 5)
+    return y.reshape(B, sh.out_ch, sh.lat_h, sh.lat_w).numpy()
+
+
+@pytest.mark.parametrize("kind", ["dit", "mmdit", "video"])
+def test_final_layer_matches_torch_composition(kind):
+    if kind == "dit":
+        sh = small_dit()
+    elif kind == "mmdit":
+        sh = small_mmdit()
+    else:
+        sh = small_mmdit(lat_f=2, lat_h=4, lat_w=6, patch_t=1, rope_dims=3)
+    W = weights64(sh, seed=11, scale=5.0)
+    tok = rnd(sh.batch_model, sh.tokens, sh.hidden, scale=2.0) + 0.7
+    c = rnd(sh.batch_model, sh.hidden, scale=3.0)
+    out = model.final_layer(W, sh, tok, c)
+    np.testing.assert_allclose(out, torch_final(W, sh, tok, c), rtol=1e-11, atol=1e-11)
+    assert out.shape == (sh.batch_model, sh.out_ch) + sh.latent_dims[2:]
+    # the layer normalises each token: an affine change of a token's values
+    # (positive scale) moves the output only through LayerNorm's eps = 1e-6
+    # (relative 1e-7 at these variances)
+    tok2 = tok * 3.0 + 11.0
+    if sh.arch == "mmdit":
+        tok2[:, :sh.txt_tokens] = 1e6   # text rows never reach the head
+    np.testing.assert_allclose(model.final_layer(W, sh, tok2, c), out, rtol=0, atol=2e-6 * np.abs(out).max())
+
+
+def test_step_update_uses_the_first_in_ch_channels_of_the_head():
+    """A learned-sigma head (2 * in_ch channels): DDIM on the guided first
+    in_ch channels; whatever the other channels hold, the latent does not
+    move with them, and with eps equal to the true noise every step lands on
+    the data.  Guidance combines [cond ; uncond] before the channel slice."""
+    sh = small_dit(in_ch=4, out_ch=8, lat_h=4, lat_w=4, batch=2)
+    N = 50
+    ab = sampler.ddim_alpha_bar()
+    ts = sampler.ddim_timesteps(N)
+    x0, eps = rnd(2, 4, 4, 4), rnd(2, 4, 4, 4)
+    x = np.sqrt(ab[ts[0]]) * x0 + np.sqrt(1 - ab[ts[0]]) * eps
+    s = sh.cfg_scale
+    for i in range(N):
+        garbage = rnd(4, 4, 4, 4, scale=1e3)
+        # cond half = eps + d, uncond half = eps + d * (s / (s - 1)): guided = eps
+        d = rnd(2, 4, 4, 4)
+        head = np.concatenate([np.concatenate([eps + d, eps + d * s / (s - 1)]), garbage], axis=1)
+        x = sampler.step_update(sh, x, head, N, i)
+    np.testing.assert_allclose(x, x0, rtol=1e-8, atol=1e-8)
+
+
+def test_step_update_euler_on_the_velocity_channels():
+    sh = small_mmdit(in_ch=4, out_ch=4, lat_h=4, lat_w=4)
+    x = rnd(1, 4, 4, 4)
+    v = rnd(1, 4, 4, 4)
+    N = 10
+    got = sampler.step_update(sh, x, v, N, 3)
+    np.testing.assert_allclose(got, x - v / N, rtol=1e-13, atol=1e-13)
+    sh8 = small_mmdit(in_ch=4, out_ch=8, lat_h=4, lat_w=4)
+    head = np.concatenate([v, rnd(1, 4, 4, 4, scale=1e3)], axis=1)
+    np.testing.assert_allclose(sampler.step_update(sh8, x, head, N, 3), got, rtol=1e-13, atol=1e-13)
