@@ -1,16 +1,23 @@
 """Benchmark of the FeatFix cached sampling path on GB300.
 
 One bench step = one whole cached sampling run (featfix_sample) of the
-DiT-XL/2-shaped bf16 workload: 28 blocks, hidden 1152, 16 heads x 72,
-MLP 4608, 32x32x4 latent with patch 2 (256 tokens), batch 8 doubled to 16 by
-classifier-free guidance, 50 DDIM steps, order-2 Taylor draft, full refresh
-every 5 steps, 8 fixed sites -- every row of the hot path (exact blocks,
-drafts, paid checks with forwarding, final layer and sampler) runs each step.
+HunyuanVideo-1.5-shaped bf16 workload, the largest of the five: 54 dual-stream
+MMDiT blocks, hidden 2048, 16 heads x 128, MLP 8192, 3-D rotary embedding,
+9 x 30 x 53 video tokens + 256 text tokens (14566), batch 1, 50 Euler steps,
+order-1 Taylor draft, full refresh every 5 steps, 12 fixed sites -- every row
+of the hot path (exact blocks, drafts, paid checks with forwarding, final
+layer and sampler) runs each step.  ``--workload dit_xl2`` (and flux, qwen)
+bench the other shapes.
 
 Metric: denoising steps per second (50 per sampling run), whole job over all
 ranks.  Inputs stay resident in HBM for ``value``; ``e2e`` repeats the
-measurement through featfix_sample_host with pinned host buffers (labels in,
-final latent out) inside the timed region.
+measurement through featfix_sample_host with pinned host buffers
+(conditioning in, final latent out) inside the timed region.
+
+Rooflines: a second timed region of the same sampling runs brackets every
+launch of each kernel class (tensor-core GEMM, attention, draft, paid check)
+with CUDA events and divides its algorithmic work by the summed time;
+``roofline`` is the class with the most time, ``rooflines`` all four.
 
 Multi-GPU: replicas only (independent samples per GPU, no collective on the
 data path); the barrier and max-over-ranks timing use torch.distributed.
@@ -35,7 +42,9 @@ if ROOT not in sys.path:
 
 METRIC = "cached-DiT denoise steps/s on 1 GB300; % of bf16 TC peak / HBM roofline"
 UNIT = "denoise steps/s"
-WORKLOAD = "dit_xl2"
+WORKLOAD = "hunyuan"
+NOMINAL_TFLOPS = 2250.0    # GB300 dense bf16 datasheet figure
+NOMINAL_GBS = 8000.0       # HBM3e, about 8 TB/s
 
 
 def parse():
@@ -47,6 +56,7 @@ def parse():
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--mode", default="featfix", choices=["featfix", "verify", "exact_only", "vanilla"])
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-leg", type=int, default=0, help=argparse.SUPPRESS)   # internal: oracle timing process
     p.add_argument("--sweep", choices=["resolution"], default=None,
                    help="instead of the headline line: one line per FLUX resolution (512^2, 768^2, 1024^2) with "
                         "sampling rate and device memory")
@@ -144,87 +154,159 @@ class ClockSampler:
 # CPU oracle baseline (bounded sample, extrapolated)
 # ----------------------------------------------------------------------------
 
-def oracle_sample_time(wl, W64, cond64, budget_s=20.0):
+FIT_ABOVE_FLOPS = 0.5e12   # exact blocks above this are timed on token-reduced copies
+
+
+def token_reduced_shapes(sh):
+    """Two copies of a shape with about 1/8 and 1/4 of its image tokens
+    (fewer video frames, or fewer patch rows of an image); same weights."""
+    from paper_2607_27842_gb300 import synthetic as syn
+    if sh.lat_f > 0:
+        f1 = max(sh.patch_t, (sh.lat_f // 8) // sh.patch_t * sh.patch_t)
+        return [syn.reduced(sh, lat_f=f1), syn.reduced(sh, lat_f=2 * f1)]
+    h1 = max(sh.patch, (sh.lat_h // 8) // sh.patch * sh.patch)
+    return [syn.reduced(sh, lat_h=h1), syn.reduced(sh, lat_h=2 * h1)]
+
+
+def oracle_sample_time(wl, W, cond64, budget_s=20.0):
     """Seconds of one whole sampling run of the oracle, extrapolated from
-    timed pieces: one exact block, one drafted block, one paid check's
-    discrepancy, the per-step conditioning/embedding/final layer/sampler."""
+    timed pieces by the plan's counts: the per-step conditioning, embedding,
+    final layer and sampler update; one exact block; one drafted block; one
+    paid check's discrepancy.  An exact block of more than 0.5 TFLOP is timed
+    on two copies of the workload with about 1/8 and 1/4 of its tokens and
+    extrapolated as a*T + b*T^2 (the projections grow linearly, attention
+    quadratically with the token count T)."""
     import numpy as np
     import oracle
     sh = wl.shape
     L = sh.n_layers
-    kind, keff = oracle.schedule.build_plan(wl.steps, L, wl.refresh, wl.K, wl.sites, "featfix")
+    kind, _ = oracle.schedule.build_plan(wl.steps, L, wl.refresh, wl.K, wl.sites, "featfix")
     n_exact = sum(k != oracle.schedule.DRAFT for row in kind for k in row)
     n_draft = sum(k != oracle.schedule.EXACT for row in kind for k in row)   # sites form the draft too
     n_site = sum(k == oracle.schedule.SITE for row in kind for k in row)
+    txt = cond64 if sh.arch == "mmdit" else None
+    labels = cond64 if sh.arch == "dit" else None
     x = oracle.noise.initial_latent(1, sh).astype(np.float64)
     t0 = time.perf_counter()
     xm = np.concatenate([x, x]) if sh.cfg else x
-    c = oracle.model.cond_vector(W64, 500.0, labels=cond64, batch=sh.batch_model)
-    tok = oracle.model.embed_tokens(W64, sh, xm)
-    out = oracle.model.final_layer(W64, sh, tok, c)
-    x = oracle.sampler.step_update(sh, x, out, wl.steps, 0)
+    c = oracle.model.cond_vector(W, 500.0, labels=labels, batch=sh.batch_model)
+    tok = oracle.model.embed_tokens(W, sh, xm, txt=txt)
+    out = oracle.model.final_layer(W, sh, tok, c)
+    oracle.sampler.step_update(sh, x, out, wl.steps, 0)
     t_step = time.perf_counter() - t0
-    reps_e, t_exact = 0, 0.0
-    while reps_e < 1 or (t_exact < budget_s * 0.6 and reps_e < 3):
-        t0 = time.perf_counter()
-        h = oracle.model.exact_block(W64, sh, reps_e % L, tok, c)
-        t_exact += time.perf_counter() - t0
-        reps_e += 1
-    hist = [(5, h - tok), (0, (h - tok) * 0.5), (-5, (h - tok) * 0.25)]
-    reps_d, t_draft = 0, 0.0
-    while reps_d < 3:
-        t0 = time.perf_counter()
+
+    pre = oracle.model.block_prefix(sh, 0)
+    for name in [n for n in W.keys() if n.startswith(pre)]:
+        W[name]                      # make the timed block's weights before timing it
+
+    def exact_once(shape):
+        u = np.ascontiguousarray(np.resize(tok, (sh.batch_model, shape.tokens, sh.hidden)))
+        t1 = time.perf_counter()
+        h = oracle.model.exact_block(W, shape, 0, u, c)
+        return time.perf_counter() - t1, h
+
+    if oracle.flops.block_flops(sh, 0) <= FIT_ABOVE_FLOPS:
+        reps, t_sum = 0, 0.0
+        while reps < 1 or (t_sum < budget_s * 0.6 and reps < 3):
+            dt, h = exact_once(sh)
+            t_sum += dt
+            reps += 1
+        t_exact = t_sum / reps
+        inc = h - tok
+        how = "%d exact block(s) at full size" % reps
+    else:
+        small = token_reduced_shapes(sh)
+        (d1, _), (d2, _) = exact_once(small[0]), exact_once(small[1])
+        T1, T2, T = small[0].tokens, small[1].tokens, sh.tokens
+        b = (d2 / T2 - d1 / T1) / (T2 - T1)
+        a = d1 / T1 - b * T1
+        if b < 0:
+            a, b = d2 / T2, 0.0
+        t_exact = a * T + b * T * T
+        inc = tok * 0.125
+        how = ("2 exact blocks at %d and %d of the %d tokens, extrapolated as a*T + b*T^2 (%.2f s / %.2f s timed, "
+               "%.1f s at full size)" % (T1, T2, T, d1, d2, t_exact))
+    hist = [(5, inc), (0, inc * 0.5), (-5, inc * 0.25)]
+    t_draft = 0.0
+    for _ in range(2):
+        t1 = time.perf_counter()
         hd = oracle.draft.draft(tok, hist[:wl.K + 1], 7, wl.K)
-        t_draft += time.perf_counter() - t0
-        reps_d += 1
-    t0 = time.perf_counter()
-    oracle.featfix.rel_l1(hd, h)
-    oracle.featfix.rel_l2(hd, h)
-    t_log = time.perf_counter() - t0
-    total = (wl.steps * t_step + n_exact * t_exact / reps_e + n_draft * t_draft / reps_d + n_site * t_log)
-    sample = ("%d exact block(s), %d draft(s), 1 discrepancy, 1 embed+final+sampler step of the %s workload, timed "
-              "and extrapolated by the plan's counts (%d exact, %d drafts, %d checks, %d steps)"
-              % (reps_e, reps_d, sh.name, n_exact, n_draft, n_site, wl.steps))
+        t_draft += (time.perf_counter() - t1) / 2
+    t1 = time.perf_counter()
+    oracle.featfix.rel_l1(hd, tok)
+    oracle.featfix.rel_l2(hd, tok)
+    t_log = time.perf_counter() - t1
+    total = wl.steps * t_step + n_exact * t_exact + n_draft * t_draft + n_site * t_log
+    sample = ("%s, 2 drafts, 1 discrepancy and 1 conditioning+embed+final+sampler step of the %s workload, "
+              "extrapolated by the plan's counts (%d exact blocks, %d drafts, %d checks, %d steps)"
+              % (how, sh.name, n_exact, n_draft, n_site, wl.steps))
     return total, sample
 
 
-def cpu_threads():
-    try:
-        from threadpoolctl import threadpool_info
-        info = threadpool_info()
-        if info:
-            return max(i.get("num_threads", 1) for i in info)
-    except Exception:
-        pass
-    return os.cpu_count() or 1
-
-
-def oracle_inputs(wl, device="cpu"):
+def lazy_oracle_inputs(wl, source=None):
+    """Float64 oracle weights made block by block on access (the large
+    workloads' float64 weights do not fit host memory) and the conditioning."""
     from paper_2607_27842_gb300 import synthetic as syn
-    w = syn.make_weights(wl.shape, seed=0, device=device)
-    return syn.oracle_weights(w), syn.oracle_cond(wl.shape, syn.make_cond(wl.shape, seed=2))
+    W = syn.LazyOracleWeights(wl.shape, seed=0, source=source, prefetch=False)
+    return W, syn.oracle_cond(wl.shape, syn.make_cond(wl.shape, seed=2))
+
+
+def cpu_leg(args, wl):
+    """Internal: time the oracle sample in this process (the thread count is
+    fixed by the parent through the BLAS environment) and print one JSON line."""
+    W, cond64 = lazy_oracle_inputs(wl)
+    t, sample = oracle_sample_time(wl, W, cond64, budget_s=10.0)
+    print(json.dumps({"seconds": t, "sample": sample, "threads": args.cpu_leg}), flush=True)
+
+
+def start_cpu_leg(wl, threads):
+    """The oracle timing as a separate interpreter (not forked from a process
+    that holds a CUDA context) with its BLAS limited to `threads` threads."""
+    env = dict(os.environ)
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[k] = str(threads)
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    return subprocess.Popen([sys.executable, os.path.abspath(__file__), "--workload", wl.shape.name,
+                             "--cpu-leg", str(threads)], stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True,
+                            env=env, cwd=ROOT)
+
+
+def finish_cpu_leg(proc, wl, timeout_s=600):
+    try:
+        out, err = proc.communicate(timeout=timeout_s)
+        rec = json.loads(out.strip().splitlines()[-1])
+        return {"value": wl.steps / rec["seconds"], "unit": UNIT, "cores": rec["threads"], "kind": "oracle",
+                "sample": rec["sample"]}
+    except Exception as e:  # reported, never fatal for the GPU number
+        proc.kill()
+        return {"value": None, "unit": UNIT, "cores": None, "kind": "oracle", "sample": "failed: %s" % e}
+
+
+def all_cores():
+    return os.cpu_count() or 1
 
 
 def run_reference(args, wl, rank):
     if rank != 0:
         return
-    W64, cond64 = oracle_inputs(wl)
-    oracle_sample_time(wl, W64, cond64, budget_s=2.0)   # untimed: first-touch of the weights
+    W, cond64 = lazy_oracle_inputs(wl)
+    for _ in range(args.warmup):
+        oracle_sample_time(wl, W, cond64, budget_s=2.0)
     times = []
     sample = ""
     for _ in range(args.steps):
-        t, sample = oracle_sample_time(wl, W64, cond64, budget_s=5.0)
+        t, sample = oracle_sample_time(wl, W, cond64, budget_s=2.0)
         times.append(t)
     t = statistics.median(times)
     value = wl.steps / t
-    cores = cpu_threads()
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(wl),
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "config": dict(workload_config(wl), mode=args.mode, parallelism="replicas x%d" % args.gpus),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": all_cores(), "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
-            "note": "CPU oracle (float64 numpy) on the host cores, extrapolated per sampling run"}
+            "note": "CPU oracle (float64 numpy) on the host cores; each step times a bounded sample of one "
+                    "sampling run and extrapolates it"}
     print(json.dumps(line), flush=True)
 
 
@@ -249,15 +331,28 @@ def job_rate(units_per_rank, world, seconds):
     return units_per_rank * world / seconds
 
 
-def profile_traffic():
-    """DRAM bytes per launch of the dominant kernel from the committed ncu
-    summary, when it was taken on the current kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", "gemm_tc_dit_xl2.md")
+KERNELS = {   # kernel class -> (kernel, bound, the sources its profile summary was taken on)
+    "gemm": ("k_gemm_tc / k_gemm_tc2 (tcgen05, all linear layers of the path)", "tensor",
+             ("ff_gemm_tc.cu", "ff_tc.cuh", "ff_common.cuh")),
+    "attention": ("k_attn_tc (tcgen05 flash attention)", "tensor", ("ff_attention_tc.cu", "ff_tc.cuh", "ff_common.cuh")),
+    "draft": ("k_draft", "hbm", ("ff_elementwise.cu", "ff_common.cuh")),
+    "verify": ("k_verify (paid check, forwarding)", "hbm", ("ff_elementwise.cu", "ff_common.cuh")),
+}
+
+
+def source_digest(files):
     src = b""
-    for f in ("ff_gemm_tc.cu", "ff_tc.cuh", "ff_common.cuh"):
+    for f in files:
         with open(os.path.join(ROOT, "paper_2607_27842_gb300", "csrc", f), "rb") as fh:
             src += fh.read()
-    digest = hashlib.sha256(src).hexdigest()[:16]
+    return hashlib.sha256(src).hexdigest()[:16]
+
+
+def profile_traffic(kclass, workload):
+    """DRAM bytes per launch of a kernel class on a workload from its committed
+    ncu summary (profiles/<class>_<workload>.md), when that summary was taken
+    on the current kernel sources (else None)."""
+    path = os.path.join(ROOT, "profiles", "%s_%s.md" % (kclass, workload))
     try:
         txt = open(path).read()
     except Exception:
@@ -268,7 +363,32 @@ def profile_traffic():
             tr = float(line.split(":")[1])
         if line.startswith("kernel_source_sha256_16:"):
             hsh = line.split(":")[1].strip()
-    return tr if hsh == digest else None
+    return tr if hsh == source_digest(KERNELS[kclass][2]) else None
+
+
+def roofline(kclass, kt, wl, steps):
+    """Achieved rate of a kernel class over the second timed region against
+    the measured peak (sustained bf16 for tensor work: the kernels run inside a
+    seconds-long step) and against the nominal GB300 figures."""
+    hbm, tf_burst, tf_sus, src = peaks()
+    ms, n, work = kt[kclass]
+    kernel, bound, _ = KERNELS[kclass]
+    if bound == "tensor":
+        ach = (work / (ms / 1e3)) / 1e12 if ms > 0 else 0.0
+        r = {"bound": "tensor", "kernel": kernel, "achieved": ach, "peak": tf_sus, "unit": "TFLOP/s",
+             "frac": ach / tf_sus, "peak_kind": "bf16_tflops_sustained (%s)" % src,
+             "frac_of_burst_peak": ach / tf_burst, "peak_nominal": NOMINAL_TFLOPS,
+             "frac_vs_nominal": ach / NOMINAL_TFLOPS}
+    else:
+        ach = (work / (ms / 1e3)) / 1e9 if ms > 0 else 0.0
+        r = {"bound": "hbm", "kernel": kernel, "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+             "peak_kind": "hbm_gbs copy (%s)" % src, "peak_nominal": NOMINAL_GBS, "frac_vs_nominal": ach / NOMINAL_GBS}
+    r.update({"traffic": profile_traffic(kclass, wl.shape.name), "launches": n, "ms_total": ms,
+              "work_per_launch": work / n if n else 0.0,
+              "work_unit": "FLOP (2*M*N*K, 4*B*H*N^2*d)" if bound == "tensor" else "bytes ((K_eff+3)*E*b, ...)",
+              "region": "second timed region: the same %d sampling runs with CUDA events on the context stream "
+                        "around every launch of the class (event nodes inside the replayed graph)" % steps})
+    return r
 
 
 def run_sweep(args):
@@ -317,17 +437,23 @@ def run_sweep(args):
 
 def main():
     args = parse()
+    from paper_2607_27842_gb300 import synthetic as syn
+    wl = syn.workload(args.workload)
+    if args.cpu_leg:
+        cpu_leg(args, wl)
+        return
     if args.sweep:
         run_sweep(args)
         return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    from paper_2607_27842_gb300 import synthetic as syn
-    wl = syn.workload(args.workload)
     if args.impl == "reference":
         run_reference(args, wl, rank)
         return
+    want_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    # the one-core oracle leg runs beside the GPU work (one host core of many)
+    leg1 = start_cpu_leg(wl, 1) if want_cpu else None
     import torch
     dist = None
     if world > 1:
@@ -372,7 +498,7 @@ def main():
     logs, counters = ff.featfix_get_log(ctx)   # synchronises and checks the watchdog
 
     # ---- timed region 2: CUDA events around every launch of each kernel class ----
-    timed_classes = ("gemm", "draft", "attention", "verify")
+    timed_classes = tuple(KERNELS)
     for k in timed_classes:
         ff.featfix_kernel_timing(ctx, k, True)
     ff.featfix_sample(ctx, 999, wl.steps, cond, lat)      # untimed: rebuilds the graph with the event nodes
@@ -401,47 +527,25 @@ def main():
     value = job_rate(args.steps * wl.steps, world, ms_max / 1e3)
     e2e = job_rate(args.steps * wl.steps, world, e2e_max)
 
-    hbm, tf_burst, tf_sus, src = peaks()
-    g_ms, g_n, g_work = kt["gemm"]
-    achieved = (g_work / (g_ms / 1e3)) / 1e12 if g_ms > 0 else 0.0
-    traffic = profile_traffic()
-    d_ms, d_n, d_work = kt["draft"]
-    draft_gbs = (d_work / (d_ms / 1e3)) / 1e9 if d_ms > 0 else 0.0
-    a_ms, a_n, a_work = kt["attention"]
-    v_ms, v_n, v_work = kt["verify"]
+    rl = {k: roofline(k, kt, wl, args.steps) for k in timed_classes}
+    dominant = max(("gemm", "attention"), key=lambda k: kt[k][0])
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_max / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "bf16", "data": "synthetic", "config": dict(workload_config(wl), mode=args.mode,
-                                                            parallelism="replicas x%d" % world),
+        "dtype": "bf16" if sh.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": dict(workload_config(wl), mode=args.mode, parallelism="replicas x%d" % world),
         "e2e": {"value": e2e, "unit": UNIT, "h2d_bytes_per_step": int(cond_h.numel() * cond_h.element_size()),
                 "d2h_bytes_per_step": int(out_h.numel() * out_h.element_size())},
         "gpu_launches": int(launches),
-        "roofline": {"bound": "tensor", "kernel": "k_gemm_tc (tcgen05, all linear layers of the path)",
-                     "region": "second timed region of the same %d sampling runs with CUDA events on the context "
-                               "stream around every launch of the kernel (inside the replayed graph)" % args.steps,
-                     "achieved": achieved, "peak": tf_sus, "unit": "TFLOP/s", "frac": achieved / tf_sus,
-                     "peak_kind": "bf16_tflops_sustained (%s)" % src, "traffic": traffic,
-                     "launches": g_n, "ms_total": g_ms},
-        "secondary": {
-            "draft": {"bound": "hbm", "achieved": draft_gbs, "peak": hbm, "unit": "GB/s",
-                      "frac": draft_gbs / hbm, "launches": d_n, "ms_total": d_ms},
-            "attention": {"achieved_tflops": (a_work / (a_ms / 1e3)) / 1e12 if a_ms > 0 else 0.0,
-                          "launches": a_n, "ms_total": a_ms},
-            "verify": {"achieved_gbs": (v_work / (v_ms / 1e3)) / 1e9 if v_ms > 0 else 0.0, "launches": v_n,
-                       "ms_total": v_ms},
-            "counters": counters},
+        "roofline": dict(rl[dominant], kclass=dominant),
+        "rooflines": rl,
+        "counters": counters,
         "clocks": clk,
     }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        try:
-            W64 = syn.oracle_weights({k: v.cpu() for k, v in weights.items()})
-            t, sample = oracle_sample_time(wl, W64, syn.oracle_cond(sh, cond.cpu()))
-            line["cpu_baseline"] = {"value": wl.steps / t, "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
-                                    "sample": sample}
-        except Exception as e:  # reported, never fatal for the GPU number
-            line["cpu_baseline"] = {"value": None, "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
-                                    "sample": "failed: %s" % e}
+    if want_cpu:
+        one_core = finish_cpu_leg(leg1, wl)
+        line["cpu_baseline"] = finish_cpu_leg(start_cpu_leg(wl, all_cores()), wl)
+        line["cpu_baseline_1core"] = one_core
     ff.featfix_destroy(ctx)
     if rank == 0:
         print(json.dumps(line), flush=True)

@@ -287,8 +287,20 @@ FEATFIX_API featfix_status featfix_plan_build_blocks(int steps, int n_layers, co
 /* Debug capture: during later trajectories, copy block `layer`'s incoming
  * state u and its forwarded output at step `step` into dev_in / dev_out
  * (device, B_model*N_tot*C elements of the model dtype, row layout of
- * featfix_token_row).  Up to 32 captures; step < 0 clears them all.        */
+ * featfix_token_row).  Up to 64 captures (of either kind below); step < 0
+ * clears them all.                                                           */
 FEATFIX_API featfix_status featfix_debug_capture(featfix_ctx* ctx, int step, int layer, void* dev_in, void* dev_out);
+
+/* Debug capture of the refresh history a draft reads (Eq. 2's finite
+ * differences are formed from these increments): during later trajectories,
+ * when block `layer` is drafted or paid-checked at step `step`, copy the
+ * first min(n, K_eff + 1) increments h^f - u of its history, newest first,
+ * as the block's draft reads them, into dev_slots[0..n-1] (device, each
+ * B_model*N_tot*C elements of the model dtype, row layout of
+ * featfix_token_row).  Nothing is copied when the block is exact at that
+ * step.  1 <= n <= 4.  Errors: INVALID_ARG for a bad layer, n or pointer.    */
+FEATFIX_API featfix_status featfix_debug_capture_history(featfix_ctx* ctx, int step, int layer,
+                                                         void* const* dev_slots, int n);
 
 /* Run the exact block B_l(u; t_step, c) (Eq. 1) on a caller state: dev_in,
  * dev_out as for featfix_debug_capture, dev_cond as for featfix_step.

@@ -24,6 +24,8 @@ struct Capture {
   int step, layer;
   void* in;
   void* out;
+  void* hist[4];   // history entries the block's draft reads, newest first
+  int nhist;
 };
 
 struct TimedLaunch {
@@ -750,9 +752,17 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
       y = (x == ctx->xa) ? ctx->xb : ctx->xa;
     };
     for (int l = 0; l < L; ++l) {
-      for (auto& cp : ctx->caps)
-        if (cp.step == i && cp.layer == l && cp.in) FF_CK(cudaMemcpyAsync(cp.in, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
       const unsigned char kind = ctx->kinds[(size_t)i * L + l];
+      for (auto& cp : ctx->caps) {
+        if (cp.step != i || cp.layer != l) continue;
+        if (cp.in) FF_CK(cudaMemcpyAsync(cp.in, x, bytes, cudaMemcpyDeviceToDevice, ctx->st));
+        if (cp.nhist > 0 && kind != FEATFIX_PLAN_EXACT) {
+          block_weights(l);
+          const Hist4 hp = hist_ptrs(ctx, l, nt);
+          for (int j = 0; j < std::min(cp.nhist, nt); ++j)
+            FF_CK(cudaMemcpyAsync(cp.hist[j], hp.p[j], bytes, cudaMemcpyDeviceToDevice, ctx->st));
+        }
+      }
       const int bslot = (ctx->bhead[l] + 1) % ctx->S;  // block l's next ring slot
       if (kind == FEATFIX_PLAN_EXACT) {
         void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, bslot) : nullptr;
@@ -1313,7 +1323,21 @@ featfix_status featfix_debug_capture(featfix_ctx* ctx, int step, int layer, void
   }
   if (layer < 0 || layer >= ctx->L || (!dev_in && !dev_out)) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "bad capture");
   if (ctx->caps.size() >= 64) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "too many captures");
-  ctx->caps.push_back({step, layer, dev_in, dev_out});
+  ctx->caps.push_back({step, layer, dev_in, dev_out, {nullptr, nullptr, nullptr, nullptr}, 0});
+  graph_reset(ctx);
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_debug_capture_history(featfix_ctx* ctx, int step, int layer, void* const* dev_slots, int n) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (step < 0 || layer < 0 || layer >= ctx->L || n < 1 || n > 4 || !dev_slots)
+    return fail(ctx, FEATFIX_ERR_INVALID_ARG, "bad history capture");
+  for (int j = 0; j < n; ++j)
+    if (!dev_slots[j]) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "bad history capture");
+  if (ctx->caps.size() >= 64) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "too many captures");
+  Capture cp = {step, layer, nullptr, nullptr, {nullptr, nullptr, nullptr, nullptr}, n};
+  for (int j = 0; j < n; ++j) cp.hist[j] = dev_slots[j];
+  ctx->caps.push_back(cp);
   graph_reset(ctx);
   return FEATFIX_OK;
 }

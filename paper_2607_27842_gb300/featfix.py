@@ -77,6 +77,7 @@ SIGNATURES = {
     "featfix_plan_build_blocks": (_I, [_I, _I, _P(_I), _I, _I, _P(Site), _I, _I, ctypes.c_uint, _P(_I), _P(_D)]),
     "featfix_debug_capture": (_I, [_VP, _I, _I, _VP, _VP]),
     "featfix_debug_block": (_I, [_VP, _I, _I, _VP, _VP, _VP]),
+    "featfix_debug_capture_history": (_I, [_VP, _I, _I, _P(_VP), _I]),
     "featfix_token_row": (_LL, [_P(ModelDesc), _I, _I]),
     "featfix_kernel_timing": (_I, [_VP, _I, _I]),
     "featfix_kernel_time": (_I, [_VP, _I, _P(_D), _P(_LL), _P(_D)]),
@@ -310,32 +311,13 @@ def featfix_plan_build(steps, n_layers, refresh, draft_order, sites, mode="featf
     return kinds.reshape(steps, n_layers), keff, w.reshape(steps, 4)
 
 
-def featfix_set_forward_mask(ctx, axis, mask=None):
-    """Partial forwarding at FeatFix sites: axis MASK_TOKENS / MASK_CHANNELS
-    with a 0/1 mask, or MASK_NONE (whole-block forwarding)."""
-    import numpy as np
-    if mask is None:
-        _check(lib().featfix_set_forward_mask(ctx, int(axis), None, 0), ctx)
-        return
-    m = np.ascontiguousarray(np.asarray(mask, dtype=np.uint8))
-    _check(lib().featfix_set_forward_mask(ctx, int(axis), m.ctypes.data_as(_P(ctypes.c_ubyte)), int(m.size)), ctx)
-
-
-def featfix_plan_build_blocks(steps, n_layers, refresh, draft_order, sites, mode="featfix", flags=0):
-    """Host-only per-block draft plan: (k_eff [steps, L], weights [steps, L, 4])."""
-    import numpy as np
-    ref = (_I * max(len(refresh), 1))(*[int(r) for r in refresh])
-    sa, ns = _sites_arr(sites)
-    keff = np.zeros(steps * n_layers, dtype=np.int32)
-    w = np.zeros(steps * n_layers * 4, dtype=np.float64)
-    m = MODES[mode] if isinstance(mode, str) else int(mode)
-    _check(lib().featfix_plan_build_blocks(int(steps), int(n_layers), ref, len(refresh), int(draft_order), sa, ns, m,
-                                           int(flags), keff.ctypes.data_as(_P(_I)), w.ctypes.data_as(_P(_D))))
-    return keff.reshape(steps, n_layers), w.reshape(steps, n_layers, 4)
-
-
 def featfix_debug_capture(ctx, step, layer, dev_in, dev_out):
     _check(lib().featfix_debug_capture(ctx, int(step), int(layer), _ptr(dev_in), _ptr(dev_out)), ctx)
+
+
+def featfix_debug_capture_history(ctx, step, layer, dev_slots):
+    arr = (_VP * len(dev_slots))(*[_ptr(t) for t in dev_slots])
+    _check(lib().featfix_debug_capture_history(ctx, int(step), int(layer), arr, len(dev_slots)), ctx)
 
 
 def featfix_debug_block(ctx, step, layer, dev_in, dev_out, cond):

@@ -124,18 +124,27 @@ SHAPES = {
 }
 
 
-# FLUX at lower resolutions (latent 64x64 / 96x96 for 512^2 / 768^2 images,
-# 1024 / 2304 image tokens) with the FLUX schedule: the resolution sweep.
-RESOLUTIONS = {"flux_512": 64, "flux_768": 96}
+# Variants of the large workloads with fewer image tokens, each at full depth
+# and width with its base workload's schedule:
+#   flux_512 / flux_768  FLUX at 512^2 / 768^2 images (latent 64x64 / 96x96,
+#                        1024 / 2304 image tokens): the resolution sweep, and
+#                        flux_512 the FLUX parity workload
+#   qwen_512             Qwen-Image at 512^2 (1024 image tokens + 256 text,
+#                        guidance batch 2)
+#   hunyuan_3f           HunyuanVideo with 3 of the 9 latent frames
+#                        (3x30x53 = 4770 video tokens + 256 text)
+# The parity workloads are the sizes at which a whole float64 oracle
+# trajectory finishes in about an hour on eight host cores.
+VARIANTS = {"flux_512": ("flux", dict(lat_h=64, lat_w=64)), "flux_768": ("flux", dict(lat_h=96, lat_w=96)),
+            "qwen_512": ("qwen", dict(lat_h=64, lat_w=64)), "hunyuan_3f": ("hunyuan", dict(lat_f=3))}
 
 
 def workload(name):
     """The schedule of each workload: draft order, refresh interval, sites."""
-    if name in RESOLUTIONS:
-        base = workload("flux")
-        side = RESOLUTIONS[name]
-        return Workload(reduced(base.shape, name=name, lat_h=side, lat_w=side), base.steps, base.K, base.refresh,
-                        base.sites)
+    if name in VARIANTS:
+        base_name, over = VARIANTS[name]
+        base = workload(base_name)
+        return Workload(reduced(base.shape, name=name, **over), base.steps, base.K, base.refresh, base.sites)
     s = SHAPES[name]
     if name == "tiny":
         return Workload(s, 10, 1, (0, 3, 6, 9), ((4, 2), (7, 1)))
@@ -159,21 +168,33 @@ def torch_dtype(shape):
     return torch.float32 if shape.dtype == "f32" else torch.bfloat16
 
 
-def make_weights(shape, seed=0, device="cpu", names=None):
+def make_weights(shape, seed=0, device="cpu", names=None, to=None):
     """Random-init weights: every tensor N(0, 0.02) from its own seeded
     generator (seed * 1000003 + index), stored in the model dtype.
-    ``names`` restricts generation to a subset (same values)."""
+    ``names`` restricts generation to a subset (same values).  ``to`` moves
+    each tensor to that device as soon as it is made (CPU-generated values
+    on a GPU without a host copy of the whole model).  On the CPU the
+    tensors are made by several threads, each from its own generator, so
+    the values do not depend on the thread count."""
+    import concurrent.futures
+    import os
     import torch
-    out = {}
     want = None if names is None else set(names)
-    for idx, (name, dims) in enumerate(weight_spec(shape)):
-        if want is not None and name not in want:
-            continue
+    jobs = [(idx, name, dims) for idx, (name, dims) in enumerate(weight_spec(shape))
+            if want is None or name in want]
+
+    def one(job):
+        idx, name, dims = job
         g = torch.Generator(device=device)
         g.manual_seed(seed * 1000003 + idx)
-        t = torch.randn(dims, generator=g, device=device, dtype=torch.float32) * WEIGHT_STD
-        out[name] = t.to(torch_dtype(shape)).contiguous()
-    return out
+        t = (torch.randn(dims, generator=g, device=device, dtype=torch.float32) * WEIGHT_STD)
+        t = t.to(torch_dtype(shape)).contiguous()
+        return name, (t if to is None else t.to(to))
+
+    if str(device) == "cpu" and len(jobs) > 1:
+        with concurrent.futures.ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
+            return dict(ex.map(one, jobs))
+    return dict(one(j) for j in jobs)
 
 
 def make_cond(shape, seed=2, device="cpu"):
@@ -211,3 +232,106 @@ def oracle_cond(shape, cond):
     if shape.arch == "dit":
         return np.asarray(cond.cpu().numpy(), dtype=np.int64)
     return to_numpy64(cond)
+
+
+def block_group(name):
+    """Weights are grouped per block ("blk3.", "dual3.", "single7.");
+    the embedding / conditioning / final-layer tensors form group ""."""
+    head = name.split(".", 1)[0]
+    if head.startswith(("blk", "dual", "single")):
+        return head + "."
+    return ""
+
+
+class LazyOracleWeights:
+    """float64 numpy weights made on first access, for models whose float64
+    weights do not fit host memory (the MMDiT workloads hold 5-20 G
+    parameters).  The values are those of ``make_weights(shape, seed)`` on the
+    CPU generator, or of the torch tensors in ``source`` when given.
+
+    Kept in memory: the non-block tensors, the most recently used block in
+    float64, and model-dtype copies of blocks while their total stays under
+    ``cache_bytes``.  Using block l starts a background thread preparing
+    block l + 1, since the oracle walks the blocks in order."""
+
+    def __init__(self, shape, seed=0, source=None, cache_bytes=0, prefetch=True):
+        import threading
+        self.shape, self.seed, self.source = shape, seed, source
+        self.cache_bytes = cache_bytes
+        self.prefetch = prefetch
+        self.spec = dict(weight_spec(shape))
+        self.groups = {}
+        for name in self.spec:
+            self.groups.setdefault(block_group(name), []).append(name)
+        self.order = [g for g in self.groups if g]
+        self.lock = threading.Lock()
+        self.low = {}          # group -> {name: model-dtype torch tensor}
+        self.low_bytes = 0
+        self.cur = {}          # group -> {name: float64 array}; the global group and at most two blocks
+        self.pending = {}      # group -> thread preparing it
+        self.cur[""] = self._make64("")
+
+    def _make_low(self, group):
+        names = self.groups[group]
+        if self.source is not None:
+            return {n: self.source[n].detach().cpu() for n in names}
+        return make_weights(self.shape, seed=self.seed, names=names)
+
+    def _make64(self, group):
+        with self.lock:
+            low = self.low.get(group)
+        if low is None:
+            low = self._make_low(group)
+            size = sum(t.numel() * t.element_size() for t in low.values())
+            with self.lock:
+                if group and self.low_bytes + size <= self.cache_bytes:
+                    self.low[group] = low
+                    self.low_bytes += size
+        return {n: to_numpy64(t) for n, t in low.items()}
+
+    def _prepare(self, group):
+        import threading
+        out = {}
+        def work():
+            out.update(self._make64(group))
+        th = threading.Thread(target=work)
+        th.result = out
+        th.start()
+        self.pending[group] = th
+
+    def _group(self, group):
+        if group in self.cur:
+            return self.cur[group]
+        th = self.pending.pop(group, None)
+        if th is not None:
+            th.join()
+            data = th.result
+        else:
+            data = self._make64(group)
+        for g in [g for g in self.cur if g]:
+            del self.cur[g]
+        self.cur[group] = data
+        if self.prefetch:
+            nxt = self.order[(self.order.index(group) + 1) % len(self.order)]
+            for g in [g for g in self.pending if g != nxt]:
+                self.pending.pop(g).join()
+            if nxt not in self.pending and nxt != group:
+                self._prepare(nxt)
+        return data
+
+    def __getitem__(self, name):
+        if name not in self.spec:
+            raise KeyError(name)
+        return self._group(block_group(name))[name]
+
+    def __contains__(self, name):
+        return name in self.spec
+
+    def keys(self):
+        return self.spec.keys()
+
+    def __iter__(self):
+        return iter(self.spec)
+
+    def __len__(self):
+        return len(self.spec)

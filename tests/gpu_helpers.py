@@ -23,27 +23,31 @@ def tol_latent(shape):
     return 1e-4 if shape.dtype == "f32" else 5e-2
 
 
-def log_close(got, ref, dtype):
-    """Logged discrepancy (Eq. 4 / rel-L2) of a free-running trajectory.
-
-    fp32: relative 1e-3.  bf16: h_d and h_f are stored in bf16, whose unit
-    roundoff 2^-8 adds rounding noise of that relative size to ||h_d - h_f||
-    -- as large as the discrepancy itself at these sites -- so the bound is
-    5% of the value plus 2^-8 absolute."""
-    if dtype == "f32":
-        return abs(got - ref) <= 1e-3 * abs(ref)
-    return abs(got - ref) <= 0.05 * abs(ref) + 2.0 ** -8
+def tol_log(shape):
+    """Logged discrepancy (Eq. 4 and its L2 analogue) against the oracle's
+    evaluated on the GPU's own tensors: 1e-4 relative in fp32 mode, 2e-2 in
+    bf16 mode.  Both sides then start from the same stored values (incoming
+    state u, the history increments the draft reads, the exact output h^f),
+    so only fp32 against fp64 arithmetic separates them."""
+    return 1e-4 if shape.dtype == "f32" else 2e-2
 
 
 class Case:
     """One model + schedule on cuda:0 with the matching oracle inputs."""
 
-    def __init__(self, wl, seed=0, weights_on_gpu=False):
+    def __init__(self, wl, seed=0, weights_on_gpu=False, keep_host=True):
+        """weights_on_gpu: drawn by the GPU generator (other values than the
+        oracle's CPU generator; for tests that compare on captured tensors).
+        keep_host=False: CPU-generated values moved to the GPU tensor by
+        tensor, with no host copy kept (the large models)."""
         self.wl = wl
         self.sh = sh = wl.shape
         self.dev = torch.device("cuda:0")
         if weights_on_gpu:
             self.w = syn.make_weights(sh, seed=seed, device=self.dev)
+            self._w_cpu = None
+        elif not keep_host:
+            self.w = syn.make_weights(sh, seed=seed, to=self.dev)
             self._w_cpu = None
         else:
             self._w_cpu = syn.make_weights(sh, seed=seed)
@@ -104,6 +108,60 @@ class Case:
                                   wl.steps, wl.refresh if refresh is None else refresh, wl.K,
                                   wl.sites if sites is None else sites, mode, hook=hook,
                                   site_updates_history=site_updates_history, forward_mask=forward_mask)
+
+    def capture_sites(self, mode="featfix", flags=0):
+        """Register captures at every paid check of the schedule: the
+        incoming state, the forwarded output and the history increments the
+        site's draft reads.  Returns {(step, layer): (u, out, [hist...])}."""
+        wl, sh = self.wl, self.sh
+        keff, _ = ff.featfix_plan_build_blocks(wl.steps, sh.n_layers, wl.refresh, wl.K, wl.sites, mode, flags)
+        bufs = {}
+        for (i, l) in wl.sites:
+            hist = [self.act_buffer() for _ in range(int(keff[i, l]) + 1)]
+            u, out = self.act_buffer(), self.act_buffer()
+            ff.featfix_debug_capture(self.ctx, i, l, u, out)
+            ff.featfix_debug_capture_history(self.ctx, i, l, hist)
+            bufs[(i, l)] = (u, out, hist)
+        return bufs
+
+    def check_logs_teacher_forced(self, bufs, logs, mode="featfix", site_updates_history=False):
+        """Every logged discrepancy against Eq. 4 (and its L2 analogue)
+        evaluated by the oracle on the GPU's own captured tensors: the draft
+        h^d formed by the oracle's Taylor series (Eq. 2) from the captured
+        history increments and rounded to the model dtype (the block output
+        as it would be forwarded), h^f the forwarded output (FeatFix) or the exact
+        block recomputed from the captured u (Verify; the GPU path is
+        deterministic, so this is the h^f the check used)."""
+        wl, sh = self.wl, self.sh
+        got = {(e["step"], e["layer"]): e for e in logs}
+        assert sorted(got) == sorted(bufs)
+        tol = tol_log(sh)
+        worst = 0.0
+        for (i, l), (u, out, hist) in bufs.items():
+            if mode == "featfix":
+                hf_dev = out
+            else:
+                hf_dev = self.act_buffer()
+                ff.featfix_debug_block(self.ctx, i, l, u, hf_dev, self.cond)
+                torch.cuda.synchronize()
+            steps = [r for r in wl.refresh if r <= i]
+            if site_updates_history:
+                steps += [s for (s, ll) in wl.sites if ll == l and s < i]
+            steps = sorted(steps, reverse=True)[:len(hist)]
+            u64, hf = self.to_logical(u), self.to_logical(hf_dev)
+            h = [(s, self.to_logical(r)) for s, r in zip(steps, hist)]
+            # Eq. 4 compares block outputs; in bf16 mode they are stored in
+            # bf16, so the draft enters the discrepancy as it would be
+            # forwarded: rounded to the model dtype
+            hd = oracle.draft.draft(u64, h, i, wl.K)
+            if sh.dtype == "bf16":
+                hd = torch.from_numpy(hd).to(torch.bfloat16).double().numpy()
+            for key, fn in (("rel_l1", oracle.featfix.rel_l1), ("rel_l2", oracle.featfix.rel_l2)):
+                ref = fn(hd, hf)
+                err = abs(got[(i, l)][key] - ref) / ref
+                worst = max(worst, err)
+                assert err <= tol, ((i, l), key, got[(i, l)][key], ref)
+        return worst
 
     def close(self):
         ff.featfix_destroy(self.ctx)

@@ -9,7 +9,7 @@ import torch
 import oracle
 from paper_2607_27842_gb300 import featfix as ff, synthetic as syn
 
-from .gpu_helpers import Case, log_close, rel_l2
+from .gpu_helpers import Case, rel_l2
 
 pytestmark = pytest.mark.gpu
 
@@ -27,9 +27,10 @@ def test_full_depth_trajectory_matches_oracle(cuda):
         x_ref, logs_ref, cnt_ref = c.oracle_run("featfix", seed=1)
         assert rel_l2(lat.cpu().numpy(), x_ref) < 5e-2
         assert {k: cnt[k] for k in cnt_ref} == cnt_ref == {"refresh_steps": 10, "paid_checks": 8, "forwarded": 8}
-        for g, r in zip(logs, logs_ref):
-            assert (g["step"], g["layer"]) == (r["step"], r["layer"])
-            assert log_close(g["rel_l2"], r["rel_l2"], "bf16"), (g, r)
+        assert [(g["step"], g["layer"]) for g in logs] == [(r["step"], r["layer"]) for r in logs_ref]
+        bufs = c.capture_sites("featfix")
+        c.sample(seed=1)
+        c.check_logs_teacher_forced(bufs, ff.featfix_get_log(c.ctx)[0], "featfix")
     finally:
         c.close()
 
