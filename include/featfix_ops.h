@@ -63,9 +63,10 @@ FEATFIX_API featfix_status featfix_op_verify(int dtype, void* dev_u, const void*
  *  - No cudaMalloc, cudaFree or other allocating routine is called.  Every
  *    GPU that loads the library holds the 16 KiB array until the process
  *    exits.
- *  - The first call on a device looks up the array's device address (with
- *    that device current) and caches it; make that first call before any
- *    stream capture on the device.
+ *  - Every call looks up the array's device address with the calling
+ *    thread's current device; the first call on a device may load the
+ *    library's module there, so make that first call before any stream
+ *    capture on the device.
  *  - A call needs featfix_op_verify_workspace(n) bytes of the array (one
  *    32-byte partial per 8-CTA cluster, at most 4 CTAs per SM); if that is
  *    more than 16 KiB (a GPU with more than 1024 SMs) the call returns

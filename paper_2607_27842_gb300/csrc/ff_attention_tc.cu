@@ -166,6 +166,40 @@ __device__ __forceinline__ float ex2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// packed pairs of fp32 (one 64-bit register pair): a.x + 2^32 * a.y
+__device__ __forceinline__ unsigned long long f2u(float a, float b) {
+  return (unsigned long long)__float_as_uint(a) | ((unsigned long long)__float_as_uint(b) << 32);
+}
+__device__ __forceinline__ unsigned long long ffma2(unsigned long long a, unsigned long long b, unsigned long long c) {
+  unsigned long long r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ unsigned long long fadd2(unsigned long long a, unsigned long long b) {
+  unsigned long long r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ float lo_f(unsigned long long x) { return __uint_as_float((unsigned)x); }
+__device__ __forceinline__ float hi_f(unsigned long long x) { return __uint_as_float((unsigned)(x >> 32)); }
+
+// 16 pairs of S (v[2e], v[2e + 1]) -> exp2(s * scale - m) as bf16 pairs,
+// their sum added to the packed accumulators
+__device__ __forceinline__ void exp_pairs16(const float* v, unsigned long long sc2, unsigned long long nm2,
+                                            unsigned long long (&acc2)[4], uint32_t (&pk)[16]) {
+#pragma unroll
+  for (int e = 0; e < 16; ++e) {
+    const unsigned long long x = ffma2(f2u(v[2 * e], v[2 * e + 1]), sc2, nm2);
+    const float p0 = ex2(lo_f(x)), p1 = ex2(hi_f(x));
+    acc2[e & 3] = fadd2(acc2[e & 3], f2u(p0, p1));
+    __nv_bfloat162 t2 = __floats2bfloat162_rn(p0, p1);
+    pk[e] = *reinterpret_cast<uint32_t*>(&t2);
+  }
+}
+__device__ __forceinline__ float acc_total(const unsigned long long (&acc2)[4]) {
+  const unsigned long long a = fadd2(fadd2(acc2[0], acc2[1]), fadd2(acc2[2], acc2[3]));
+  return lo_f(a) + hi_f(a);
+}
 
 __device__ __forceinline__ void tma_load3(const CUtensorMap* tm, uint64_t* bar, void* dst, int x, int y, int z) {
   asm volatile(
@@ -257,7 +291,7 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int nk = 0, nv = 0;
+      int nk = 0, nv = 0, q_last = -1;
       bool ok = true;
       for (int it = 0; it < ipc && ok && item_live(it); ++it) {
         // the next item's Q waits for the previous item's last S MMAs
@@ -268,6 +302,7 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
           for (int bx = 0; bx < C::NBOX; ++bx)
             tma_load3(&tmQKV, q_full, sQ + i * C::TILE + bx * C::BOX, 64 * bx, h, qs.row0);
         }
+        q_last = it;
         for (int j = 0; j < nkv; ++j) {
           const int jj = it * nkv + j;
           const SegTile ks = seg_tile(a, b, j);
@@ -296,6 +331,13 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
         const int j = nv - 1 - k;
         const unsigned long long t0 = gtimer();
         while (!mbar_try(&v_full[j % C::VST], (j / C::VST) & 1))
+          if (gtimer() - t0 > WAIT_LIMIT_NS) { atomicOr(&g_attn_watchdog, 2u); break; }
+      }
+      // and the last item's query tiles (phase q_last of q_full; on the
+      // normal path the MMA warp has already seen it complete)
+      if (q_last >= 0) {
+        const unsigned long long t0 = gtimer();
+        while (!mbar_try(q_full, q_last & 1))
           if (gtimer() - t0 > WAIT_LIMIT_NS) { atomicOr(&g_attn_watchdog, 2u); break; }
       }
     }
@@ -389,6 +431,92 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
       // registers; two query tiles: the row is held in registers.
       float v[QT == 1 ? 1 : AKV];
       float mx[16];
+      if constexpr (QT == 2) {
+        // Speculative softmax: exponentials against the running reference
+        // m while S streams in from TMEM, P stored as it is made.  They are
+        // the lazy-rescale result whenever no exponent exceeds 2^8, which a
+        // tile sum <= 256 guarantees; otherwise (and on the first tile) the
+        // row max is taken from the registers, O is rescaled if the max
+        // grew by more than 2^8, and P is recomputed.
+        const unsigned long long sc2 = f2u(scale_log2, scale_log2);
+        bool need = true;
+        float lt = 0.f;
+        if (j > 0) {
+          const unsigned long long nm2 = f2u(-m, -m);
+          unsigned long long acc2[4] = {0ull, 0ull, 0ull, 0ull};
+          tmem_ld32_async(s_col, v);
+          tmem_wait32(v);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            // S columns [32 (k + 1), 32 (k + 2)) load while chunk k is
+            // finished; P chunk k goes to columns [16 k, 16 k + 16), which
+            // hold S already read
+            if (k + 1 < 4) tmem_ld32_async(s_col + (uint32_t)(32 * (k + 1)), v + 32 * (k + 1));
+            if (valid < AKV) {
+#pragma unroll
+              for (int e = 0; e < 32; ++e)
+                if (32 * k + e >= valid) v[32 * k + e] = -INFINITY;
+            }
+            uint32_t pk[16];
+            exp_pairs16(v + 32 * k, sc2, nm2, acc2, pk);
+            tmem_st16u(s_col + (uint32_t)(16 * k), pk);
+            if (k + 1 < 4) tmem_wait32(v + 32 * (k + 1));
+          }
+          lt = acc_total(acc2);
+          need = __any_sync(0xffffffffu, !(lt <= 256.0f));   // also a non-finite sum
+        } else {
+          tmem_ld64w(s_col, v);
+          tmem_ld64w(s_col + 64, v + 64);
+          if (valid < AKV) {
+#pragma unroll
+            for (int e = 0; e < AKV; ++e)
+              if (e >= valid) v[e] = -INFINITY;
+          }
+        }
+        float alpha = 1.0f;
+        if (need) {
+#pragma unroll
+          for (int e = 0; e < 16; ++e)
+            mx[e] = max3f(max3f(v[e], v[e + 16], v[e + 32]), max3f(v[e + 48], v[e + 64], v[e + 80]),
+                          fmaxf(v[e + 96], v[e + 112]));
+#pragma unroll
+          for (int e = 0; e < 5; ++e) mx[e] = max3f(mx[e], mx[e + 5], mx[e + 10]);
+          mx[0] = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[15]), mx[0]);
+          const float m_new = fmaxf(m, mx[0] * scale_log2);
+          const bool grow = m_new > m + RESCALE_LOG2;  // always on the first tile
+          if (__any_sync(0xffffffffu, grow)) {
+            alpha = grow ? ex2(m - m_new) : 1.0f;
+            // O_i holds every update through tile j - 1: s_full[i] for tile
+            // j arrived after them
+            if (j >= 1) {
+#pragma unroll
+              for (int c = 0; c < C::DK / 16; ++c) {
+                float o[16];
+                tmem_ld16(o_col + (uint32_t)(c * 16), o);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) o[e] *= alpha;
+                tmem_st16(o_col + (uint32_t)(c * 16), o);
+              }
+            }
+            if (grow) m = m_new;
+            tmem_st_wait();   // the speculative P stores land before their recomputation
+            const unsigned long long nm2 = f2u(-m, -m);
+            unsigned long long acc2[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              uint32_t pk[16];
+              exp_pairs16(v + 32 * k, sc2, nm2, acc2, pk);
+              tmem_st16u(s_col + (uint32_t)(16 * k), pk);
+            }
+            lt = acc_total(acc2);
+          }
+        }
+        l = l * alpha + lt;
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(&p_ready[i]);
+        continue;
+      }
       if constexpr (QT == 1) {
 #pragma unroll
         for (int e = 0; e < 16; ++e) mx[e] = -INFINITY;

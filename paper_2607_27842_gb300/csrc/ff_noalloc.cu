@@ -4,8 +4,6 @@
 #include "featfix_ops.h"
 #include "ff_common.cuh"
 
-#include <mutex>
-
 namespace {
 
 // Scratch of the verify reduction: one 4-double partial per 8-CTA cluster
@@ -14,26 +12,16 @@ namespace {
 constexpr size_t kNoallocScratchBytes = FEATFIX_VERIFY_NOALLOC_SCRATCH_BYTES;
 static __device__ __align__(256) double g_verify_scratch[kNoallocScratchBytes / sizeof(double)];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-void* g_scratch_addr[kMaxDevices] = {};
-
 // Device address of the array on the current device.  Host code only sees a
-// host-side stand-in under the array's name, so the address is looked up
-// once per device (with that device current) and cached.
+// host-side stand-in under the array's name, so the address is looked up with
+// the device current -- on every call: after a device reset or a re-created
+// primary context the module may be loaded at another address, and once the
+// module is loaded the lookup is cheap.
 cudaError_t scratch_address(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_verify_scratch);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_verify_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = p;
-  }
-  *out = g_scratch_addr[dev];
+  *out = p;
   return cudaSuccess;
 }
 
