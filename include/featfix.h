@@ -302,6 +302,16 @@ FEATFIX_API featfix_status featfix_debug_capture(featfix_ctx* ctx, int step, int
 FEATFIX_API featfix_status featfix_debug_capture_history(featfix_ctx* ctx, int step, int layer,
                                                          void* const* dev_slots, int n);
 
+/* Failure-detection test hook (the paper has no counterpart).  Launches, on
+ * the context stream, one CTA that takes tensor memory as the tensor-core
+ * GEMM does and then waits, with the GEMM's bounded wait, on an mbarrier
+ * that nothing arrives on.  After limit_ns (1 us .. 1 s) the wait gives up,
+ * raises the watchdog flag a stuck GEMM or attention kernel raises, and the
+ * CTA frees its tensor memory and returns: nothing traps and the context
+ * stays usable.  The next featfix_get_log then reports FEATFIX_ERR_CUDA
+ * (and clears the flag).  Errors: INVALID_ARG for a limit out of range.     */
+FEATFIX_API featfix_status featfix_debug_watchdog_probe(featfix_ctx* ctx, unsigned long long limit_ns);
+
 /* Run the exact block B_l(u; t_step, c) (Eq. 1) on a caller state: dev_in,
  * dev_out as for featfix_debug_capture, dev_cond as for featfix_step.
  * Requires a schedule (for t_step).  Ordered on the context stream.         */

@@ -275,9 +275,12 @@ struct FwdMix {
   const unsigned char* cmask;
   int C;
 };
+// done_ctr: a zeroed counter owned by the caller turns the reduction into
+// one launch (the last cluster sums the partials and resets the counter);
+// without it a second one-block launch sums them.
 cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
                           int write_draft, double* sums, void* ws, cudaStream_t s,
-                          const FwdMix* mix = nullptr);
+                          const FwdMix* mix = nullptr, unsigned int* done_ctr = nullptr);
 cudaError_t launch_ln_mod(DType dt, const void* x, void* out, long long rows, int C, const float* shift,
                           const float* scale, int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s);
 // Sinusoidal features of S model times (device array) -> [S, 256] in dt.
@@ -303,6 +306,7 @@ cudaError_t gemm_simt(DType dt, int M, int N, int K, const void* A, int lda, con
 cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, int ldw, const EpiArgs& e,
                     cudaStream_t s);
 unsigned int gemm_tc_watchdog_take();
+cudaError_t watchdog_probe(unsigned long long limit_ns, cudaStream_t s);
 
 // attention over the token-row layout (see featfix_token_row)
 struct AttnArgs {

@@ -174,7 +174,8 @@ template <class T, int NT>
 __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_THREADS)
     k_verify(T* __restrict__ u, Hist4 h, float w0, float w1, float w2, float w3, const T* hf,
              long long n, int write_draft, double* __restrict__ partials, T* mix,
-             const unsigned char* __restrict__ rmask, const unsigned char* __restrict__ cmask, int C) {
+             const unsigned char* __restrict__ rmask, const unsigned char* __restrict__ cmask, int C,
+             unsigned int* done_ctr, double* __restrict__ sums) {
   pdl_trigger();
   pdl_wait();
   constexpr int V = VecN<T>::n;
@@ -228,13 +229,36 @@ __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_
   }
   cg::cluster_group cluster = cg::this_cluster();
   cluster.sync();
-  if (cluster.block_rank() == 0 && threadIdx.x < 4) {
-    double t = 0.0;
-    for (unsigned r = 0; r < cluster.num_blocks(); ++r) {
-      const double* rb = cluster.map_shared_rank(bsum, r);
-      t += rb[threadIdx.x];
+  if (cluster.block_rank() == 0 && threadIdx.x < 32) {
+    if (threadIdx.x < 4) {
+      double t = 0.0;
+      for (unsigned r = 0; r < cluster.num_blocks(); ++r) {
+        const double* rb = cluster.map_shared_rank(bsum, r);
+        t += rb[threadIdx.x];
+      }
+      partials[(size_t)(blockIdx.x / VERIFY_CLUSTER) * 4 + threadIdx.x] = t;
+      __threadfence();
     }
-    partials[(size_t)(blockIdx.x / VERIFY_CLUSTER) * 4 + threadIdx.x] = t;
+    // With a completion counter the last cluster to finish sums every
+    // cluster's partials in index order (the same order whichever cluster
+    // is last) and resets the counter for the next launch.
+    if (done_ctr) {
+      __syncwarp();
+      const unsigned int nclusters = gridDim.x / VERIFY_CLUSTER;
+      unsigned int last = 0;
+      if (threadIdx.x == 0) last = atomicAdd(done_ctr, 1u) == nclusters - 1 ? 1u : 0u;
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (last) {
+        __threadfence();
+        if (threadIdx.x < 4) {
+          const volatile double* vp = partials;
+          double t = 0.0;
+          for (unsigned k = 0; k < nclusters; ++k) t += vp[(size_t)k * 4 + threadIdx.x];
+          sums[threadIdx.x] = t;
+        }
+        if (threadIdx.x == 0) *done_ctr = 0u;
+      }
+    }
   }
   cluster.sync();
 }
@@ -251,7 +275,8 @@ __global__ void k_verify_finish(const double* __restrict__ partials, int nparts,
 
 template <class T>
 static cudaError_t verify_t(void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
-                           int write_draft, double* sums, void* ws, cudaStream_t s, const FwdMix* fm) {
+                           int write_draft, double* sums, void* ws, cudaStream_t s, const FwdMix* fm,
+                           unsigned int* done_ctr) {
   const int grid = verify_grid(n);
   double* parts = reinterpret_cast<double*>(ws);
   T* up = reinterpret_cast<T*>(u);
@@ -262,23 +287,24 @@ static cudaError_t verify_t(void* u, const Hist4& h, const float* w, int nt, con
   const int C = fm ? fm->C : 1;
   if (mx && (C <= 0 || C % VecN<T>::n != 0 || (!rm && !cm) || n % C != 0)) return cudaErrorInvalidValue;
   switch (nt) {
-    case 1: launch_pdl(k_verify<T, 1>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C); break;
-    case 2: launch_pdl(k_verify<T, 2>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C); break;
-    case 3: launch_pdl(k_verify<T, 3>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C); break;
-    case 4: launch_pdl(k_verify<T, 4>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C); break;
+    case 1: launch_pdl(k_verify<T, 1>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C, done_ctr, sums); break;
+    case 2: launch_pdl(k_verify<T, 2>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C, done_ctr, sums); break;
+    case 3: launch_pdl(k_verify<T, 3>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C, done_ctr, sums); break;
+    case 4: launch_pdl(k_verify<T, 4>, grid, VERIFY_THREADS, 0, s, up, h, w[0], w[1], w[2], w[3], fp, n, write_draft, parts, mx, rm, cm, C, done_ctr, sums); break;
     default: return cudaErrorInvalidValue;
   }
   cudaError_t e = launched();
-  if (e != cudaSuccess) return e;
+  if (e != cudaSuccess || done_ctr) return e;
   launch_pdl(k_verify_finish, 1, 32, 0, s, parts, grid / VERIFY_CLUSTER, sums);
   return launched();
 }
 
 cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
-                          int write_draft, double* sums, void* ws, cudaStream_t s, const FwdMix* mix) {
+                          int write_draft, double* sums, void* ws, cudaStream_t s, const FwdMix* mix,
+                          unsigned int* done_ctr) {
   if (n <= 0) return cudaErrorInvalidValue;
-  return dt == F32 ? verify_t<float>(u, h, w, nt, hf, n, write_draft, sums, ws, s, mix)
-                   : verify_t<bf16>(u, h, w, nt, hf, n, write_draft, sums, ws, s, mix);
+  return dt == F32 ? verify_t<float>(u, h, w, nt, hf, n, write_draft, sums, ws, s, mix, done_ctr)
+                   : verify_t<bf16>(u, h, w, nt, hf, n, write_draft, sums, ws, s, mix, done_ctr);
 }
 
 // ---------------------------------------------------------------------------

@@ -851,6 +851,47 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
   return launched();
 }
 
+// ---------------------------------------------------------------------------
+// Watchdog probe (failure-detection test hook): one CTA takes TMEM like the
+// GEMM does, then waits with the GEMM's bounded wait on an mbarrier that
+// nothing arrives on.  The wait gives up after limit_ns, raises the same
+// watchdog flag a stuck GEMM raises, and the CTA frees its TMEM and returns.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(64, 1) k_watchdog_probe(unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_flag;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);   // one arrival expected; none comes
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(&tmem_slot)), "r"(32)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+  if (lane == 0) mbar_wait<true>(&bar, 0, &abort_flag, &g_watchdog, limit_ns);
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(32) : "memory");
+  }
+}
+
+cudaError_t watchdog_probe(unsigned long long limit_ns, cudaStream_t s) {
+  k_watchdog_probe<<<1, 64, 0, s>>>(limit_ns);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
 unsigned int gemm_tc_watchdog_take() {
   unsigned int v = 0, z = 0;
   if (cudaMemcpyFromSymbol(&v, g_watchdog, sizeof(v)) != cudaSuccess) return 0;

@@ -660,6 +660,10 @@ featfix_status finish_step(featfix_ctx* ctx, int i, const void* x, float* latent
   return FEATFIX_OK;
 }
 
+unsigned int* verify_counter(featfix_ctx* c) {
+  return reinterpret_cast<unsigned int*>(reinterpret_cast<char*>(c->vws) + c->vws_bytes - 256);
+}
+
 void* ring_slot(featfix_ctx* c, int l, int slot) {
   return off(c->ring, ((long long)l * c->S + slot) * c->E, c->es);
 }
@@ -697,7 +701,7 @@ featfix_status verify_shadow(featfix_ctx* ctx, int i, int nt, const float* wf) {
       if (slot >= ctx->max_logs) return fail(ctx, FEATFIX_ERR_STATE, "log overflow");
       KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 3) * bytes);
       FF_CK(launch_verify(ctx->dt, ctx->shadow, hist_ptrs(ctx, l, nt), wf, nt, ctx->xa, ctx->E, 1,
-                          ctx->dsums + 4 * slot, ctx->vws, ctx->st));
+                          ctx->dsums + 4 * slot, ctx->vws, ctx->st, nullptr, verify_counter(ctx)));
       ctx->log_sites.push_back({i, l});
     } else {
       KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
@@ -788,7 +792,7 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
                              ctx->fmask_axis == FEATFIX_MASK_CHANNELS ? ctx->d_cmask : nullptr, ctx->C};
           KTimer tm(ctx, FEATFIX_KCLASS_VERIFY, (double)(nt + 2 + wr + (partial ? 1 : 0)) * bytes);
           FF_CK(launch_verify(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, y, ctx->E, wr, ctx->dsums + 4 * slot,
-                              ctx->vws, ctx->st, partial ? &fm : nullptr));
+                              ctx->vws, ctx->st, partial ? &fm : nullptr, verify_counter(ctx)));
           ctx->log_sites.push_back({i, l});
         }
         if (ctx->mode != FEATFIX_MODE_VERIFY) {
@@ -1008,10 +1012,12 @@ featfix_status schedule_buffers(featfix_ctx* ctx, int steps, int K, int mode, in
     FF_TRY(alloc(ctx, (void**)&ctx->dsums, (size_t)nlog * 4 * sizeof(double)));
     ctx->max_logs = nlog;
   }
-  const size_t need = verify_workspace_bytes(ctx->E);
+  // the partials, then the completion counter of the one-launch reduction
+  const size_t need = (verify_workspace_bytes(ctx->E) + 255) / 256 * 256 + 256;
   if (need > ctx->vws_bytes) {
     free_ptr(&ctx->vws);
     FF_TRY(alloc(ctx, &ctx->vws, need));
+    FF_CK(cudaMemsetAsync(ctx->vws, 0, need, ctx->user_st));
     ctx->vws_bytes = need;
   }
   void** tabs[] = {(void**)&ctx->d_times, (void**)&ctx->d_need, &ctx->sin_tab, &ctx->thid_tab, (void**)&ctx->temb_tab,
@@ -1325,6 +1331,13 @@ featfix_status featfix_debug_capture(featfix_ctx* ctx, int step, int layer, void
   if (ctx->caps.size() >= 64) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "too many captures");
   ctx->caps.push_back({step, layer, dev_in, dev_out, {nullptr, nullptr, nullptr, nullptr}, 0});
   graph_reset(ctx);
+  return FEATFIX_OK;
+}
+
+featfix_status featfix_debug_watchdog_probe(featfix_ctx* ctx, unsigned long long limit_ns) {
+  if (!ctx) return FEATFIX_ERR_INVALID_ARG;
+  if (limit_ns < 1000ull || limit_ns > 1000000000ull) return fail(ctx, FEATFIX_ERR_INVALID_ARG, "probe limit out of range");
+  FF_CK(watchdog_probe(limit_ns, ctx->user_st));
   return FEATFIX_OK;
 }
 

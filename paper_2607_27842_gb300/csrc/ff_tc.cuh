@@ -55,14 +55,15 @@ __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
 // suspending try_wait); false (and the CTA abort flag raised) on timeout or
 // when another role already aborted.
 template <bool SPIN = false>
-static __device__ __noinline__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, unsigned int* watchdog) {
+static __device__ __noinline__ bool mbar_wait(uint64_t* b, uint32_t parity, volatile int* abort_flag, unsigned int* watchdog,
+                                              unsigned long long limit_ns = WAIT_LIMIT_NS) {
   if (SPIN ? mbar_test(b, parity) : mbar_try(b, parity)) return true;
   const unsigned long long t0 = gtimer();
   for (uint32_t it = 1;; ++it) {
     if (SPIN ? mbar_test(b, parity) : mbar_try(b, parity)) return true;
     if ((it & 63) == 0) {
       if (*abort_flag) return false;
-      if (gtimer() - t0 > WAIT_LIMIT_NS) {
+      if (gtimer() - t0 > limit_ns) {
         *abort_flag = 1;
         atomicOr(watchdog, 1u);
         return false;

@@ -78,6 +78,7 @@ SIGNATURES = {
     "featfix_debug_capture": (_I, [_VP, _I, _I, _VP, _VP]),
     "featfix_debug_block": (_I, [_VP, _I, _I, _VP, _VP, _VP]),
     "featfix_debug_capture_history": (_I, [_VP, _I, _I, _P(_VP), _I]),
+    "featfix_debug_watchdog_probe": (_I, [_VP, ctypes.c_ulonglong]),
     "featfix_token_row": (_LL, [_P(ModelDesc), _I, _I]),
     "featfix_kernel_timing": (_I, [_VP, _I, _I]),
     "featfix_kernel_time": (_I, [_VP, _I, _P(_D), _P(_LL), _P(_D)]),
@@ -318,6 +319,10 @@ def featfix_debug_capture(ctx, step, layer, dev_in, dev_out):
 def featfix_debug_capture_history(ctx, step, layer, dev_slots):
     arr = (_VP * len(dev_slots))(*[_ptr(t) for t in dev_slots])
     _check(lib().featfix_debug_capture_history(ctx, int(step), int(layer), arr, len(dev_slots)), ctx)
+
+
+def featfix_debug_watchdog_probe(ctx, limit_ns):
+    _check(lib().featfix_debug_watchdog_probe(ctx, int(limit_ns)), ctx)
 
 
 def featfix_debug_block(ctx, step, layer, dev_in, dev_out, cond):

@@ -175,7 +175,12 @@ def make_weights(shape, seed=0, device="cpu", names=None, to=None):
     each tensor to that device as soon as it is made (CPU-generated values
     on a GPU without a host copy of the whole model).  On the CPU the
     tensors are made by several threads, each from its own generator, so
-    the values do not depend on the thread count."""
+    the values do not depend on the thread count.
+
+    CPU draws are made in float64 and rounded to float32, then to the model
+    dtype: torch's float64 normal sampler gives the same values on x86 and
+    Arm hosts, its float32 sampler (vectorised differently per
+    instruction set) does not."""
     import concurrent.futures
     import os
     import torch
@@ -187,7 +192,10 @@ def make_weights(shape, seed=0, device="cpu", names=None, to=None):
         idx, name, dims = job
         g = torch.Generator(device=device)
         g.manual_seed(seed * 1000003 + idx)
-        t = (torch.randn(dims, generator=g, device=device, dtype=torch.float32) * WEIGHT_STD)
+        if str(device) == "cpu":
+            t = (torch.randn(dims, generator=g, dtype=torch.float64) * WEIGHT_STD).to(torch.float32)
+        else:
+            t = torch.randn(dims, generator=g, device=device, dtype=torch.float32) * WEIGHT_STD
         t = t.to(torch_dtype(shape)).contiguous()
         return name, (t if to is None else t.to(to))
 
@@ -209,11 +217,12 @@ def make_cond(shape, seed=2, device="cpu"):
         if shape.cfg:
             lab = torch.cat([lab, torch.full((shape.batch,), shape.n_classes, dtype=torch.int64)])
         return lab.to(torch.int32).to(device)
-    txt = torch.randn((shape.batch, shape.txt_tokens, shape.hidden), generator=g, dtype=torch.float32)
+    # float64 draws rounded to float32 (the same values on x86 and Arm hosts)
+    txt = torch.randn((shape.batch, shape.txt_tokens, shape.hidden), generator=g, dtype=torch.float64).float()
     if shape.cfg:
         g2 = torch.Generator(device="cpu")
         g2.manual_seed(seed + 1000)
-        unc = torch.randn((shape.batch, shape.txt_tokens, shape.hidden), generator=g2, dtype=torch.float32)
+        unc = torch.randn((shape.batch, shape.txt_tokens, shape.hidden), generator=g2, dtype=torch.float64).float()
         txt = torch.cat([txt, unc])
     return txt.contiguous().to(device)
 
