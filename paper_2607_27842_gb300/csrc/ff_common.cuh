@@ -305,6 +305,11 @@ cudaError_t gemm_simt(DType dt, int M, int N, int K, const void* A, int lda, con
                       const EpiArgs& e, cudaStream_t s);
 cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, int ldw, const EpiArgs& e,
                     cudaStream_t s);
+// Two problems of the same N and K (A0 W0^T with epilogue e0 over M0 rows and
+// A1 W1^T with e1 over M1 rows, the same lda / ldw) in one persistent launch
+// where possible: the second stream's few tiles fill the wave of the first.
+cudaError_t gemm_tc_grouped(int M0, const void* A0, const void* W0, const EpiArgs& e0, int M1, const void* A1,
+                            const void* W1, const EpiArgs& e1, int N, int K, int lda, int ldw, cudaStream_t s);
 unsigned int gemm_tc_watchdog_take();
 cudaError_t watchdog_probe(unsigned long long limit_ns, cudaStream_t s);
 

@@ -114,13 +114,21 @@ __device__ __forceinline__ TileAt tile_at(const TileMap& t, int tile) {
   return {true, (u % t.num_m2) * 256, t.n_full * BN + (u / t.num_m2) * 128};
 }
 
+// Group 1 (optional, tm1.n_tiles > 0): a second problem of the same N and K
+// with its own A, W, rows and epilogue (the text stream of a two-stream
+// block beside the image stream), its tiles first in the tile list; only
+// normal tiles, no residual preloads.  In each loop body `e`, `M` and `tm`
+// name the tile's group.
 template <int BN>
 __global__ void __launch_bounds__(THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmW128, const __grid_constant__ CUtensorMap tmA256,
               const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmH,
-              const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmHB, int M, int N, int K,
-              TileMap tm, EpiArgs e) {
+              const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmHB, int M0, int N, int K,
+              const __grid_constant__ TileMap tm0, const __grid_constant__ EpiArgs e0,
+              const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+              const __grid_constant__ CUtensorMap tmO1, const __grid_constant__ CUtensorMap tmH1, int M1,
+              const __grid_constant__ TileMap tm1, const __grid_constant__ EpiArgs e1) {
   using C = Cfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -136,7 +144,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int num_tiles = tm.n_tiles;
+  const int n1 = tm1.n_tiles;
+  const int num_tiles = tm0.n_tiles + n1;
   const int num_kb = (K + BK - 1) / BK;
 
   if (threadIdx.x == 0) {
@@ -153,9 +162,13 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
-    if (tm.pre & 1) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmR) : "memory");
-    if (tm.pre & 2) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmHB) : "memory");
-    if (tm.n_tiles > tm.n_norm) {
+    if (tm0.pre & 1) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmR) : "memory");
+    if (tm0.pre & 2) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmHB) : "memory");
+    if (n1) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA1) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB1) : "memory");
+    }
+    if (tm0.n_tiles > tm0.n_norm) {
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmW128) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA256) : "memory");
     }
@@ -180,7 +193,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-        const TileAt t = tile_at<BN>(tm, tile);
+        const bool g1 = tile < n1;
+        const TileAt t = g1 ? tile_at<BN>(tm1, tile) : tile_at<BN>(tm0, tile - n1);
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
@@ -189,7 +203,10 @@ __global__ void __launch_bounds__(THREADS, 1)
           // normal: A rows -> M side, W rows -> N side; swapped: the reverse.
           // (Each call names its kernel parameter: a tensor map must stay in
           // parameter space, never be copied to local memory.)
-          if (!t.sw) {
+          if (g1) {
+            tma_load(&tmA1, &full[s], sA + s * C::A_BYTES, kb * BK, t.m0);
+            tma_load(&tmB1, &full[s], sB + s * C::B_BYTES, kb * BK, t.n0);
+          } else if (!t.sw) {
             tma_load(&tmA, &full[s], sA + s * C::A_BYTES, kb * BK, t.m0);
             tma_load(&tmB, &full[s], sB + s * C::B_BYTES, kb * BK, t.n0);
           } else {
@@ -250,7 +267,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint4 pr[4], ph[4];
     float pb = 0.f, pg0 = 0.f, pg1 = 0.f;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++tc) {
-      const TileAt t = tile_at<BN>(tm, tile);
+      const bool g1 = tile < n1;
+      const EpiArgs& e = g1 ? e1 : e0;
+      const TileMap& tm = g1 ? tm1 : tm0;
+      const int M = g1 ? M1 : M0;
+      const TileAt t = tile_at<BN>(tm, g1 ? tile : tile - n1);
       const int acc = tc & 1;
       const uint32_t aph = (tc >> 1) & 1;
       // staged epilogue: residual / history-base rows of chunk n0 into pr /
@@ -395,8 +416,13 @@ __global__ void __launch_bounds__(THREADS, 1)
           fence_async_smem();
           __syncwarp();
           if (lane == 0) {
-            tma_store(&tmO, b0, n0, t.m0 + q * 32);
-            if (e.hist_out) tma_store(&tmH, ep + 2048, n0, t.m0 + q * 32);
+            if (g1) {
+              tma_store(&tmO1, b0, n0, t.m0 + q * 32);
+              if (e.hist_out) tma_store(&tmH1, ep + 2048, n0, t.m0 + q * 32);
+            } else {
+              tma_store(&tmO, b0, n0, t.m0 + q * 32);
+              if (e.hist_out) tma_store(&tmH, ep + 2048, n0, t.m0 + q * 32);
+            }
             bulk_commit();
           }
           ++epi_cnt;
@@ -838,16 +864,69 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
       if (e.hist_out && make_store_map(&mhb, const_cast<void*>(e.hist_base), M, N, e.ldo)) tm.pre |= 2;
     }
     const int grid = (int)(t256 < g_sms ? t256 : g_sms);
+    const TileMap none = {};
     launch_pdl(k_gemm_tc<256>, grid, THREADS, Cfg<256>::SMEM, s, ma, mb, mw128, ma256, mo, mh, mr, mhb, M, N, K, tm,
-               e);
+               e, ma, mb, mo, mh, 0, none, e);
   } else {
     tm.n_full = (N + 127) / 128;
     tm.n_norm = tm.num_m * tm.n_full;
     tm.n_tiles = tm.n_norm;
     if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, 128)) return cudaErrorInvalidValue;
     const int grid = (int)(t128 < g_sms ? t128 : g_sms);
-    launch_pdl(k_gemm_tc<128>, grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, ma, mb, M, N, K, tm, e);
+    const TileMap none = {};
+    launch_pdl(k_gemm_tc<128>, grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, ma, mb, M, N, K, tm, e, ma,
+               mb, ma, mb, 0, none, e);
   }
+  return launched();
+}
+
+namespace {
+// Normal 128 x 256 tiles of one problem (N a multiple of 256) with the
+// staged TMA-store epilogue where the output allows it.
+bool group_maps(int M, int N, int K, const void* A, int lda, const void* W, int ldw, const EpiArgs& e, TileMap* tm,
+                CUtensorMap* ma, CUtensorMap* mb, CUtensorMap* mo, CUtensorMap* mh) {
+  *tm = {};
+  tm->num_m = (M + BM - 1) / BM;
+  tm->num_m2 = (M + 255) / 256;
+  tm->n_full = N / 256;
+  tm->n_norm = tm->num_m * tm->n_full;
+  tm->n_tiles = tm->n_norm;
+  if (!make_map(ma, A, M, K, lda, BM) || !make_map(mb, W, N, K, ldw, 256)) return false;
+  *mo = *ma;
+  *mh = *ma;
+  const bool aligned = !((uintptr_t)e.out & 15) && e.ldo % 8 == 0 &&
+                       (!e.hist_out || (!((uintptr_t)e.hist_out & 15) && !((uintptr_t)e.hist_base & 15)));
+  const bool gate_ok = !e.gate || ((e.seg_split <= 0 || e.rpb0 >= 32) && e.rpb1 >= 32);
+  if (!e.out_f32 && e.split_col >= N && aligned && gate_ok && make_store_map(mo, e.out, M, N, e.ldo) &&
+      (!e.hist_out || make_store_map(mh, e.hist_out, M, N, e.ldo)))
+    tm->staged = 1;
+  return true;
+}
+}  // namespace
+
+cudaError_t gemm_tc_grouped(int M0, const void* A0, const void* W0, const EpiArgs& e0, int M1, const void* A1,
+                            const void* W1, const EpiArgs& e1, int N, int K, int lda, int ldw, cudaStream_t s) {
+  if (M1 <= 0) return gemm_tc(M0, N, K, A0, lda, W0, ldw, e0, s);
+  if (M0 <= 0) return gemm_tc(M1, N, K, A1, lda, W1, ldw, e1, s);
+  if (!init_driver()) return cudaErrorNotSupported;
+  // CTA-pair reductions and column counts that need swapped tiles run as
+  // two launches
+  if ((M0 >= 2 * BM && K >= 8192) || N % 256 != 0) {
+    const cudaError_t r = gemm_tc(M1, N, K, A1, lda, W1, ldw, e1, s);
+    return r != cudaSuccess ? r : gemm_tc(M0, N, K, A0, lda, W0, ldw, e0, s);
+  }
+  if (K % 8 != 0 || lda % 8 != 0 || ldw % 8 != 0) return cudaErrorInvalidValue;
+  if (((uintptr_t)A0 & 15) || ((uintptr_t)W0 & 15) || ((uintptr_t)A1 & 15) || ((uintptr_t)W1 & 15))
+    return cudaErrorInvalidValue;
+  TileMap t0, t1;
+  CUtensorMap a0, b0, o0, h0, a1, b1, o1, h1;
+  if (!group_maps(M0, N, K, A0, lda, W0, ldw, e0, &t0, &a0, &b0, &o0, &h0) ||
+      !group_maps(M1, N, K, A1, lda, W1, ldw, e1, &t1, &a1, &b1, &o1, &h1))
+    return cudaErrorInvalidValue;
+  const long long tiles = (long long)t0.n_tiles + t1.n_tiles;
+  const int grid = (int)(tiles < g_sms ? tiles : g_sms);
+  launch_pdl(k_gemm_tc<256>, grid, THREADS, Cfg<256>::SMEM, s, a0, b0, a0, a0, o0, h0, a0, a0, M0, N, K, t0, e0, a1,
+             b1, o1, h1, M1, t1, e1);
   return launched();
 }
 

@@ -424,6 +424,18 @@ cudaError_t dense(featfix_ctx* c, int M, int N, int K, const void* A, int lda, c
   return gemm_simt(c->dt, M, N, K, A, lda, W, K, e, c->st);
 }
 
+// Two streams' layers of the same shape (image rows M0, text rows M1) in one
+// launch where the tensor-core GEMM can group them.
+cudaError_t dense2(featfix_ctx* c, int M0, const void* A0, const void* W0, const EpiArgs& e0, int M1, const void* A1,
+                   const void* W1, const EpiArgs& e1, int N, int K, int lda) {
+  if (c->dt != BF16) {
+    const cudaError_t r = dense(c, M1, N, K, A1, lda, W1, e1);
+    return r != cudaSuccess ? r : dense(c, M0, N, K, A0, lda, W0, e0);
+  }
+  KTimer tm(c, FEATFIX_KCLASS_GEMM, 2.0 * (M0 + M1) * N * (double)K);
+  return gemm_tc_grouped(M0, A0, W0, e0, M1, A1, W1, e1, N, K, lda, K, c->st);
+}
+
 EpiArgs epi(void* out, int ldo, const void* bias) {
   EpiArgs e = epi_plain(out, ldo);
   e.bias = bias;
@@ -488,48 +500,58 @@ featfix_status block_dit(featfix_ctx* ctx, int i, int l, const void* u, void* ou
 }
 
 // Exact MMDiT two-stream block: per-stream modulation and projections,
-// joint attention.  Text rows [0, Bm*Nt), image rows after.
+// joint attention.  Text rows [0, Bm*Nt), image rows after; each layer runs
+// both streams in one grouped launch (image rows as group 0, text as group 1).
 featfix_status block_dual(featfix_ctx* ctx, int i, int l, const void* u, void* out, void* hist) {
   const int C = ctx->C, M = ctx->M, es = ctx->es;
   const int wb = 10 + 20 * l;
   const auto& W = ctx->w;
   const long long rt = (long long)ctx->Bm * ctx->Nt, ri = (long long)ctx->Bm * ctx->Ni;
   const Mod mi = block_mod(ctx, i, l, 0), mt = block_mod(ctx, i, l, 1);
-  // stream s: 0 text, 1 image
+  const int ti = (int)ri, tt = (int)rt;
+  // per-stream views: s = 0 text, 1 image
+  auto rows0 = [&](int s_) { return s_ == 0 ? 0LL : rt; };
   for (int s = 0; s < 2; ++s) {
-    const long long r0 = s == 0 ? 0 : rt, rows = s == 0 ? rt : ri;
-    if (!rows) continue;
-    FF_CK(ln_mod(ctx, coff(u, r0 * C, es), off(ctx->xm, r0 * C, es), rows, s ? mi : mt, 0, 1, 0, 1,
-                 s ? ctx->Ni : ctx->Nt));
-    const int wq = s ? wb + 4 : wb + 6;
-    EpiArgs e = epi(off(ctx->qkv, r0 * 3 * C, es), 3 * C, W[wq + 1]);
-    if (s == 1 && ctx->rope) {
-      e.rope = ctx->rope; e.rope_row0 = 0; e.rope_period = ctx->Ni; e.rope_cols = 2 * C; e.rope_hd = ctx->hd;
-    }
-    FF_CK(dense(ctx, (int)rows, 3 * C, C, off(ctx->xm, r0 * C, es), C, W[wq], e));
+    const long long rows = s == 0 ? rt : ri;
+    if (rows)
+      FF_CK(ln_mod(ctx, coff(u, rows0(s) * C, es), off(ctx->xm, rows0(s) * C, es), rows, s ? mi : mt, 0, 1, 0, 1,
+                   s ? ctx->Ni : ctx->Nt));
   }
+  EpiArgs qi = epi(off(ctx->qkv, rt * 3 * C, es), 3 * C, W[wb + 5]);
+  if (ctx->rope) {
+    qi.rope = ctx->rope; qi.rope_row0 = 0; qi.rope_period = ctx->Ni; qi.rope_cols = 2 * C; qi.rope_hd = ctx->hd;
+  }
+  const EpiArgs qt = epi(ctx->qkv, 3 * C, W[wb + 7]);
+  FF_CK(dense2(ctx, ti, off(ctx->xm, rt * C, es), W[wb + 4], qi, tt, ctx->xm, W[wb + 6], qt, 3 * C, C, C));
   FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, es), off(ctx->qkv, 2 * C, es), 3 * C, ctx->att, C));
+  EpiArgs pe[2];
   for (int s = 0; s < 2; ++s) {
-    const long long r0 = s == 0 ? 0 : rt, rows = s == 0 ? rt : ri;
-    if (!rows) continue;
     const Mod& m = s ? mi : mt;
-    const int rpb = s ? ctx->Ni : ctx->Nt;
     const int wp = s ? wb + 8 : wb + 10;
-    EpiArgs e = epi(off(ctx->u1, r0 * C, es), C, W[wp + 1]);
-    e.gate = m.chunk(2, C); e.gate_stride = m.stride; e.rpb1 = rpb;
-    e.resid = coff(u, r0 * C, es); e.ld_resid = C;
-    FF_CK(dense(ctx, (int)rows, C, C, off(ctx->att, r0 * C, es), C, W[wp], e));
-    FF_CK(ln_mod(ctx, off(ctx->u1, r0 * C, es), off(ctx->xm, r0 * C, es), rows, m, 3, 4, 0, 1, rpb));
-    const int wf = s ? wb + 12 : wb + 16;
-    EpiArgs e1 = epi(off(ctx->big, r0 * M, es), M, W[wf + 1]);
-    e1.act = 1;
-    FF_CK(dense(ctx, (int)rows, M, C, off(ctx->xm, r0 * C, es), C, W[wf], e1));
-    EpiArgs e2 = epi(off(out, r0 * C, es), C, W[wf + 3]);
-    e2.gate = m.chunk(5, C); e2.gate_stride = m.stride; e2.rpb1 = rpb;
-    e2.resid = off(ctx->u1, r0 * C, es); e2.ld_resid = C;
-    if (hist) { e2.hist_base = coff(u, r0 * C, es); e2.hist_out = off(hist, r0 * C, es); }
-    FF_CK(dense(ctx, (int)rows, C, M, off(ctx->big, r0 * M, es), M, W[wf + 2], e2));
+    pe[s] = epi(off(ctx->u1, rows0(s) * C, es), C, W[wp + 1]);
+    pe[s].gate = m.chunk(2, C); pe[s].gate_stride = m.stride; pe[s].rpb1 = s ? ctx->Ni : ctx->Nt;
+    pe[s].resid = coff(u, rows0(s) * C, es); pe[s].ld_resid = C;
   }
+  FF_CK(dense2(ctx, ti, off(ctx->att, rt * C, es), W[wb + 8], pe[1], tt, ctx->att, W[wb + 10], pe[0], C, C, C));
+  for (int s = 0; s < 2; ++s) {
+    const long long rows = s == 0 ? rt : ri;
+    if (rows)
+      FF_CK(ln_mod(ctx, off(ctx->u1, rows0(s) * C, es), off(ctx->xm, rows0(s) * C, es), rows, s ? mi : mt, 3, 4, 0,
+                   1, s ? ctx->Ni : ctx->Nt));
+  }
+  EpiArgs f1[2], f2[2];
+  for (int s = 0; s < 2; ++s) {
+    const Mod& m = s ? mi : mt;
+    const int wf = s ? wb + 12 : wb + 16;
+    f1[s] = epi(off(ctx->big, rows0(s) * M, es), M, W[wf + 1]);
+    f1[s].act = 1;
+    f2[s] = epi(off(out, rows0(s) * C, es), C, W[wf + 3]);
+    f2[s].gate = m.chunk(5, C); f2[s].gate_stride = m.stride; f2[s].rpb1 = s ? ctx->Ni : ctx->Nt;
+    f2[s].resid = off(ctx->u1, rows0(s) * C, es); f2[s].ld_resid = C;
+    if (hist) { f2[s].hist_base = coff(u, rows0(s) * C, es); f2[s].hist_out = off(hist, rows0(s) * C, es); }
+  }
+  FF_CK(dense2(ctx, ti, off(ctx->xm, rt * C, es), W[wb + 12], f1[1], tt, ctx->xm, W[wb + 16], f1[0], M, C, C));
+  FF_CK(dense2(ctx, ti, off(ctx->big, rt * M, es), W[wb + 14], f2[1], tt, ctx->big, W[wb + 18], f2[0], C, M, M));
   return FEATFIX_OK;
 }
 
