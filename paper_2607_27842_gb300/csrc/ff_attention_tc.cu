@@ -654,6 +654,306 @@ __global__ void __launch_bounds__(ACfg<D, QT>::THREADS, QT == 1 ? 2 : 1)
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Sequences of at most two key tiles (256 tokens; DiT-XL/2) with a head
+// width of at most 80: one query tile at a time, two CTAs per SM, every CTA
+// taking the query tiles of one (sample, head) in turn.  The head's K and V
+// tiles are loaded once and stay resident for all of the CTA's query tiles;
+// S over all keys comes from one N = 256 MMA, so the softmax needs no online
+// rescaling (one pass for the row max, one for P).  Head widths over 64 keep
+// their last 16 columns in separate 32-byte-swizzled boxes (4 KB per tile
+// instead of a second 16 KB box), which lets Q, both K and both V tiles of a
+// 72-wide head fit two CTAs per SM.  TMEM (256 columns): S in [0, 256), P
+// over its first half, O in [128, 128 + DK) once the softmax has read S.
+// ---------------------------------------------------------------------------
+template <int D> struct ACfgShort {
+  static constexpr int DK = (D + 15) / 16 * 16;      // 64 or 80
+  static constexpr bool TAIL = DK > 64;
+  static constexpr uint32_t MAIN = 128 * 128;        // [128 rows x 64] bf16, 128-byte swizzle
+  static constexpr uint32_t TAILB = 128 * 32;        // [128 rows x 16] bf16, 32-byte swizzle
+  static constexpr uint32_t BYTES_Q = MAIN + (TAIL ? TAILB : 0);   // one tile of q, k or v
+  static constexpr int THREADS = 192;
+  static constexpr uint32_t TMEM_COLS = 256;
+  // kind::f16, D fp32, A/B bf16; S: both K-major, N set per launch (128 or
+  // 256); O: A (P) from TMEM, B (V) MN-major, N = 64 (+ 16 for the tail)
+  static constexpr uint32_t IDESC_S128 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(128 >> 3) << 17) |
+                                         ((uint32_t)(AQ >> 4) << 24);
+  static constexpr uint32_t IDESC_S256 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(256 >> 3) << 17) |
+                                         ((uint32_t)(AQ >> 4) << 24);
+  static constexpr int VN = (DK + 31) / 32 * 32;     // P V width: whole 32-column boxes (64 or 96)
+  static constexpr uint32_t IDESC_O = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((uint32_t)(VN >> 3) << 17) |
+                                      ((uint32_t)(AQ >> 4) << 24);
+  static constexpr uint32_t VBOX = 128 * 64;          // [128 keys x 32] bf16, 64-byte swizzle
+  static constexpr uint32_t VTILE = (VN / 32) * VBOX; // a V tile: VN / 32 such boxes along the head width
+};
+// shared-memory layout of the short kernel (offsets from the 1 KB-aligned base)
+struct ShortLayout {
+  static constexpr uint32_t QA = 0;          // 16 KB
+  static constexpr uint32_t QT = 16384;      // 4 KB
+  static constexpr uint32_t KA = 20480;      // 2 x 16 KB, adjacent: one 256-row K-major operand
+  static constexpr uint32_t KT = 53248;      // 2 x 4 KB, adjacent
+  static constexpr uint32_t VA = 61440;      // 2 x 24 KB: tile j, head columns 32i .. 32i + 31 at + 24 KB j + 8 KB i
+  static constexpr uint32_t BARS = 110592;   // barriers, TMEM slot, abort flag
+  static constexpr size_t SMEM = 1024 + 110592 + 256;   // two CTAs per SM
+};
+static_assert(ShortLayout::KA % 1024 == 0 && ShortLayout::VA % 1024 == 0 && ShortLayout::QT % 1024 == 0 &&
+                  ShortLayout::KT % 1024 == 0 && ShortLayout::VA + 2 * 3 * 8192 <= ShortLayout::BARS,
+              "swizzle atoms need 1 KB-aligned tiles");
+
+// K-major operand with 32-byte swizzle: 8-row groups 256 B apart
+__device__ __forceinline__ uint64_t sw32_desc(uint32_t addr) {
+  uint64_t d = (uint64_t)((addr & 0x3FFFF) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(256 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)6 << 61;
+  return d;
+}
+// MN-major operand with 64-byte swizzle: 32-element atoms along N 8 KB
+// apart (one [128 x 32] box each), 8 rows along K per 512-byte group
+__device__ __forceinline__ uint64_t sw64_desc_mn(uint32_t addr) {
+  uint64_t d = (uint64_t)((addr & 0x3FFFF) >> 4);
+  d |= (uint64_t)(8192 >> 4) << 16;
+  d |= (uint64_t)(512 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)4 << 61;
+  return d;
+}
+
+template <int D>
+__global__ void __launch_bounds__(192, 2)
+    k_attn_short(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ CUtensorMap tmTail,
+                 const __grid_constant__ CUtensorMap tmV, AttnArgs a, float scale_log2, int ipc) {
+  using C = ACfgShort<D>;
+  using L = ShortLayout;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BARS);
+  uint64_t* q_full = bars;
+  uint64_t* k_full = bars + 1;
+  uint64_t* v_full = bars + 2;
+  uint64_t* s_full = bars + 3;
+  uint64_t* p_ready = bars + 4;
+  uint64_t* o_final = bars + 5;
+  uint64_t* q_empty = bars + 6;
+  uint64_t* o_free = bars + 7;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y, b = blockIdx.z;
+  const int nkv = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;   // 1 or 2
+  auto item_live = [&](int it) { return blockIdx.x * ipc + it < nkv; };
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    mbar_init(k_full, 1);
+    mbar_init(v_full, 1);
+    mbar_init(s_full, 1);
+    mbar_init(p_ready, 128);
+    mbar_init(o_final, 1);
+    mbar_init(q_empty, 1);
+    mbar_init(o_free, 128);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmQKV) : "memory");
+    if (C::TAIL) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmTail) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmV) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(tmem_slot)),
+                 "r"(C::TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // a tile of the q (section 0), k (1) or v (2) columns of head h: its
+      // 128-byte box and, for head widths over 64, the 32-byte tail box
+      bool k_issued = false, v_issued = false;
+      int q_last = -1;
+      if (item_live(0)) {
+        mbar_expect_tx(k_full, (uint32_t)nkv * C::BYTES_Q);
+        for (int j = 0; j < nkv; ++j) {
+          const int row0 = seg_tile(a, b, j).row0;
+          tma_load3(&tmQKV, k_full, smem + L::KA + j * C::MAIN, 0, a.H + h, row0);
+          if (C::TAIL) tma_load3(&tmTail, k_full, smem + L::KT + j * C::TAILB, 64, a.H + h, row0);
+        }
+        k_issued = true;
+        for (int it = 0; it < ipc && item_live(it); ++it) {
+          if (it > 0 && !wait_a(q_empty, (it - 1) & 1, abort_flag)) break;
+          mbar_expect_tx(q_full, C::BYTES_Q);
+          const int qrow0 = seg_tile(a, b, blockIdx.x * ipc + it).row0;
+          tma_load3(&tmQKV, q_full, smem + L::QA, 0, h, qrow0);
+          if (C::TAIL) tma_load3(&tmTail, q_full, smem + L::QT, 64, h, qrow0);
+          q_last = it;
+          if (it == 0) {
+            mbar_expect_tx(v_full, (uint32_t)nkv * C::VTILE);
+            for (int j = 0; j < nkv; ++j) {
+              const int row0 = seg_tile(a, b, j).row0;
+#pragma unroll
+              for (int i = 0; i < C::VN / 32; ++i)
+                tma_load3(&tmV, v_full, smem + L::VA + j * C::VTILE + i * C::VBOX, 32 * i, 2 * a.H + h, row0);
+            }
+            v_issued = true;
+          }
+        }
+      }
+      // copies still in flight land before the CTA exits
+      auto drain = [&](uint64_t* bar, uint32_t parity) {
+        const unsigned long long t0 = gtimer();
+        while (!mbar_try(bar, parity))
+          if (gtimer() - t0 > WAIT_LIMIT_NS) { atomicOr(&g_attn_watchdog, 2u); break; }
+      };
+      if (k_issued) drain(k_full, 0);
+      if (v_issued) drain(v_full, 0);
+      if (q_last >= 0) drain(q_full, q_last & 1);
+    }
+  } else if (warp == 1) {
+    bool ok = true;
+    const uint32_t base = saddr(smem);
+    const uint32_t idesc_s = nkv > 1 ? C::IDESC_S256 : C::IDESC_S128;
+    for (int it = 0; it < ipc && ok && item_live(it); ++it) {
+      ok = wait_u(q_full, it & 1, abort_flag);
+      if (ok && it == 0) ok = wait_u(k_full, 0, abort_flag);
+      // O of the previous item is read out before S overwrites its columns
+      if (ok && it > 0) ok = wait_u(o_free, (it - 1) & 1, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      // S = Q K^T over all keys: 4 steps of 16 in the 128-byte boxes (+32 B
+      // per step inside the swizzle atom), then the 32-byte tail box
+#pragma unroll
+      for (int k = 0; k < C::DK / 16; ++k) {
+        const uint64_t ad = k < 4 ? sw128_desc(base + L::QA) + (uint64_t)(2 * k) : sw32_desc(base + L::QT);
+        const uint64_t bd = k < 4 ? sw128_desc(base + L::KA) + (uint64_t)(2 * k) : sw32_desc(base + L::KT);
+        if (elect_one()) umma(tmem, ad, bd, idesc_s, k != 0);
+      }
+      if (elect_one()) {
+        umma_commit(s_full);
+        umma_commit(q_empty);
+      }
+      ok = wait_u(p_ready, it & 1, abort_flag);
+      if (ok && it == 0) ok = wait_u(v_full, 0, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      // O = P V: keys 16k .. 16k + 15 are P columns 8k .. 8k + 7; 16 rows of
+      // key tile k / 8 (1 KB into each of its 64-byte-swizzled boxes)
+      for (int k = 0; k < 8 * nkv; ++k) {
+        const int j = k >> 3, kk = k & 7;
+        const uint64_t vd = sw64_desc_mn(base + L::VA + j * C::VTILE + (uint32_t)kk * 1024u);
+        if (elect_one()) umma_ts(tmem + 128, tmem + (uint32_t)(8 * k), vd, C::IDESC_O, k != 0);
+      }
+      if (elect_one()) umma_commit(o_final);
+    }
+  } else {
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    const uint32_t s_col = tmem + ((uint32_t)(q * 32) << 16);
+    const uint32_t o_col = s_col + 128;
+    const int valid0 = seg_tile(a, b, 0).valid;
+    const int valid1 = nkv > 1 ? seg_tile(a, b, 1).valid : 0;
+    bool ok = true;
+    for (int it = 0; it < ipc && ok && item_live(it); ++it) {
+      const SegTile qs = seg_tile(a, b, blockIdx.x * ipc + it);
+      int w = 1;
+      if (lane == 0) w = wait_a(s_full, it & 1, abort_flag) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+      tc_fence_after();
+      // pass 1: row max over the keys, 64 columns at a time
+      float mx[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e) mx[e] = -INFINITY;
+#pragma unroll
+      for (int c4 = 0; c4 < 4; ++c4) {
+        if (c4 >= 2 * nkv) break;
+        float t[64];
+        tmem_ld64w(s_col + (uint32_t)(64 * c4), t);
+        const int vt = (c4 < 2 ? valid0 : valid1) - 64 * (c4 & 1);   // valid keys in these 64 columns
+        if (vt < 64) {
+#pragma unroll
+          for (int e = 0; e < 64; ++e)
+            if (e >= vt) t[e] = -INFINITY;
+        }
+#pragma unroll
+        for (int e = 0; e < 16; ++e) mx[e] = max3f(mx[e], max3f(t[e], t[e + 16], t[e + 32]), t[e + 48]);
+      }
+#pragma unroll
+      for (int e = 0; e < 5; ++e) mx[e] = max3f(mx[e], mx[e + 5], mx[e + 10]);
+      mx[0] = max3f(max3f(mx[0], mx[1], mx[2]), max3f(mx[3], mx[4], mx[15]), mx[0]);
+      const float m = mx[0] * scale_log2;
+      // pass 2: P = exp2(s * scale - m) as bf16 pairs over the first half of
+      // S (chunk k of 32 keys -> columns 16k .. 16k + 15, already read)
+      const unsigned long long sc2 = f2u(scale_log2, scale_log2), nm2 = f2u(-m, -m);
+      unsigned long long acc2[4] = {0ull, 0ull, 0ull, 0ull};
+      float sq[2][32];
+      tmem_ld32_async(s_col, sq[0]);
+      tmem_wait32(sq[0]);
+      const int nch = 4 * nkv;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        if (k >= nch) break;
+        if (k + 1 < nch) tmem_ld32_async(s_col + (uint32_t)(32 * (k + 1)), sq[(k + 1) & 1]);
+        float* x = sq[k & 1];
+        const int vt = (k < 4 ? valid0 : valid1) - 32 * (k & 3);
+        if (vt < 32) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (e >= vt) x[e] = -INFINITY;
+        }
+        uint32_t pk[16];
+        exp_pairs16(x, sc2, nm2, acc2, pk);
+        tmem_st16u(s_col + (uint32_t)(16 * k), pk);
+        if (k + 1 < nch) tmem_wait32(sq[(k + 1) & 1]);
+      }
+      const float l = acc_total(acc2);
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(p_ready);
+      if (lane == 0) w = wait_a(o_final, it & 1, abort_flag) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+      tc_fence_after();
+      // O into registers, then TMEM is released (the next query tile's S
+      // MMA may start) before the output is written
+      float o[C::DK / 16][16];
+#pragma unroll
+      for (int c = 0; c < C::DK / 16; ++c) tmem_ld16(o_col + (uint32_t)(c * 16), o[c]);
+      tc_fence_before();
+      mbar_arrive(o_free);
+      const float inv = 1.0f / l;
+      bf16* orow = reinterpret_cast<bf16*>(a.out) + (size_t)(qs.row0 + (r < qs.valid ? r : 0)) * a.ld_out + (size_t)h * D;
+      if (r < qs.valid) {
+#pragma unroll
+        for (int c = 0; c < C::DK / 16; ++c) {
+#pragma unroll
+          for (int e = 0; e < 16; e += 8) {
+            if (c * 16 + e < D) {
+              float t8[8];
+#pragma unroll
+              for (int z = 0; z < 8; ++z) t8[z] = o[c][e + z] * inv;
+              st16(orow + c * 16 + e, t8);
+            }
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::TMEM_COLS) : "memory");
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
 std::once_flag g_once;
 int g_attn_sms = 148;
@@ -672,6 +972,8 @@ bool init_attn() {
 #define FF_ATTR(d, qt) \
   cudaFuncSetAttribute(k_attn_tc<d, qt>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ACfg<d, qt>::SMEM)
     FF_ATTR(64, 1); FF_ATTR(64, 2); FF_ATTR(72, 1); FF_ATTR(72, 2); FF_ATTR(128, 1); FF_ATTR(128, 2);
+    cudaFuncSetAttribute(k_attn_short<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ShortLayout::SMEM);
+    cudaFuncSetAttribute(k_attn_short<72>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ShortLayout::SMEM);
 #undef FF_ATTR
   });
   return g_enc != nullptr;
@@ -696,6 +998,25 @@ cudaError_t attn_tc_t(const AttnArgs& a, cudaStream_t s) {
   // tile per CTA, two CTAs per SM, longer ones two query tiles per CTA
   const int nq = (a.Nt + 127) / 128 + (a.Ni + 127) / 128;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)D);
+  if (nq <= 2 && D <= 80) {
+    // resident K / V, one N = 256 S per query tile (DiT-XL/2's 256 tokens)
+    // q / k columns 64 .. 79 (32-byte swizzle), v in 32-column boxes (64-byte swizzle)
+    CUtensorMap tt = tm, tv = tm;
+    cuuint32_t box16[3] = {16, 1, 128}, box32[3] = {32, 1, 128};
+    if (g_enc(&tt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.q), dims, strides, box16, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_32B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS ||
+        g_enc(&tv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.q), dims, strides, box32, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    const long long heads = (long long)a.H * a.B, slots = 2LL * g_attn_sms;
+    int ipc = 1;
+    while (ipc < nq && (long long)((nq + ipc - 1) / ipc) * heads > slots) ++ipc;
+    launch_pdl(k_attn_short<D <= 64 ? 64 : 72>, dim3((nq + ipc - 1) / ipc, a.H, a.B), ACfgShort<D <= 64 ? 64 : 72>::THREADS,
+               ShortLayout::SMEM, s, tm, tt, tv, a, scale_log2, ipc);
+    return launched();
+  }
   if (nq <= SHORT_KV_TILES) {
     // query tiles of one (sample, head) per CTA: as few as keep the CTAs
     // within one wave of two per SM, so the second tile's loads overlap the

@@ -207,6 +207,11 @@ def test_gemm_is_deterministic(cuda):
 ATTN_CASES = [
     # dtype, B, n_txt, n_img, heads, d
     ("bf16", 2, 0, 256, 3, 72),
+    # at most two key tiles, head width <= 80: K / V resident, one N = 256 S
+    ("bf16", 4, 0, 100, 3, 72),        # one key tile (N = 128 S), ragged
+    ("bf16", 2, 40, 60, 2, 72),        # text tile + image tile, both ragged
+    ("bf16", 2, 5, 100, 2, 64),        # head width 64 (no tail box)
+    ("bf16", 3, 0, 256, 5, 64),
     ("bf16", 1, 5, 70, 2, 128),
     ("bf16", 2, 3, 130, 2, 64),
     ("bf16", 1, 0, 200, 4, 32),
