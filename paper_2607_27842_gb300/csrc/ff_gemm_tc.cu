@@ -114,12 +114,313 @@ __device__ __forceinline__ TileAt tile_at(const TileMap& t, int tile) {
   return {true, (u % t.num_m2) * 256, t.n_full * BN + (u / t.num_m2) * 128};
 }
 
-// Group 1 (optional, tm1.n_tiles > 0): a second problem of the same N and K
+// Per-warp constants of the epilogue warps.
+struct EpiWarp {
+  uint8_t* smem;      // the 1024-aligned shared-memory base (ring first)
+  uint8_t* ep;        // the warp's 4 KB output / transpose buffer
+  uint64_t* rbar;     // per-warp residual / history-base barriers
+  uint64_t* tfull;    // accumulator-full barriers
+  volatile int* abort_flag;
+  uint32_t tmem_base;
+  int warp, lane, q, h, row, c_lo;
+};
+
+// The epilogue of one tile, inlined once per problem of the launch so that
+// every EpiArgs / TileMap field and tensor map is read from its own kernel
+// parameter (a run-time choice between two parameter structs turns every
+// field access of the inner loops into a generic load).  PLAIN: normal
+// tiles without residual preloads (the second problem of a grouped launch).
+// Returns false when the accumulator wait gave up.
+template <int BN, bool PLAIN>
+__device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, const TileMap& tm, const int M,
+                                         const int N, const TileAt t, const int acc, const uint32_t aph,
+                                         uint32_t& epi_cnt, const CUtensorMap* tmO, const CUtensorMap* tmH,
+                                         const CUtensorMap* tmR, const CUtensorMap* tmHB) {
+  using C = Cfg<BN>;
+  const int warp = W.warp, lane = W.lane, q = W.q, h = W.h, row = W.row, c_lo = W.c_lo;
+  uint8_t* const smem = W.smem;
+  uint8_t* const ep = W.ep;
+  float* const xp = reinterpret_cast<float*>(ep);
+  uint64_t* const rbar = W.rbar;
+  uint64_t* const tfull = W.tfull;
+  volatile int* const abort_flag = W.abort_flag;
+  const uint32_t tmem_base = W.tmem_base;
+  const int pre = PLAIN ? 0 : tm.pre;
+  const bool sw = !PLAIN && t.sw;
+  uint4 pr[4], ph[4];
+  float pb = 0.f, pg0 = 0.f, pg1 = 0.f;
+  // staged epilogue: residual / history-base rows of chunk n0 into pr /
+  // ph; bias and gate of column n0 + lane into pb / pg0 / pg1 (shared
+  // across the warp by shuffles: the warp's 32 rows lie in samples
+  // b_lo .. b_hi, at most two of them)
+  const int wr0 = t.m0 + q * 32;
+  const int b_lo = e.gate ? epi_batch(e, min(wr0, M - 1)) : 0;
+  const int b_hi = e.gate ? epi_batch(e, min(wr0 + 31, M - 1)) : 0;
+  auto fetch = [&](int n0) {
+    const int m = t.m0 + row;
+    const bool cin = n0 + lane < N;
+    pb = (e.bias && cin) ? __bfloat162float(reinterpret_cast<const bf16*>(e.bias)[n0 + lane]) : 0.f;
+    pg0 = (e.gate && cin) ? e.gate[(size_t)b_lo * e.gate_stride + n0 + lane] : 0.f;
+    pg1 = (e.gate && cin && b_hi != b_lo) ? e.gate[(size_t)b_hi * e.gate_stride + n0 + lane] : pg0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const bool in = m < M && n0 + 8 * k < N;
+      if (e.resid && !(pre & 1))
+        pr[k] = in ? *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.resid) +
+                                                      (size_t)m * e.ld_resid + n0 + 8 * k)
+                   : make_uint4(0, 0, 0, 0);
+      if (e.hist_out && !(pre & 2))
+        ph[k] = in ? *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.hist_base) +
+                                                      (size_t)m * e.ldo + n0 + 8 * k)
+                   : make_uint4(0, 0, 0, 0);
+    }
+  };
+  if (C::XPOSE_BYTES > 0 && tm.staged && !sw) fetch(t.n0 + c_lo);
+  int ok = 1;
+  if (lane == 0) ok = mbar_wait_g(&tfull[acc], aph, abort_flag) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  if (!ok) return false;
+  tc_fence_after();
+  // One tile per CTA: the ring's last readers (this tile's MMAs) are
+  // complete, so the warp's residual / history-base blocks (4 x 32 x 32
+  // bf16 each, 64-byte swizzle: the layout of the output blocks) come by
+  // TMA into its 8 KB slices of the ring; waited for at first use.
+  uint8_t* rsm = smem + (warp - 2) * 8192;
+  uint8_t* hsm = smem + 65536 + (warp - 2) * 8192;
+  bool pre_wait = pre != 0;
+  if (pre && lane == 0) {
+    mbar_expect_tx(&rbar[warp - 2], ((pre & 1) ? 8192u : 0u) + ((pre & 2) ? 8192u : 0u));
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int x = sw ? t.n0 + q * 32 : t.n0 + c_lo + 32 * i;
+      const int y = sw ? t.m0 + h * (BN / 2) + 32 * i : t.m0 + q * 32;
+      if (pre & 1) tma_load(tmR, &rbar[warp - 2], rsm + i * 2048, x, y);
+      if (pre & 2) tma_load(tmHB, &rbar[warp - 2], hsm + i * 2048, x, y);
+    }
+  }
+  auto pre_ready = [&]() -> bool {
+    if (!pre_wait) return true;
+    pre_wait = false;
+    int w = 1;
+    if (lane == 0) w = mbar_wait_g(&rbar[warp - 2], 0, abort_flag) ? 1 : 0;
+    return __shfl_sync(0xffffffffu, w, 0) != 0;
+  };
+  const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+  if (!sw && (C::XPOSE_BYTES == 0 || !tm.staged)) {
+    const int m = t.m0 + row;
+    for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
+      const int n0 = t.n0 + c;
+      if (n0 >= N) break;
+      float v[32];
+      tmem_ld32(tq + (uint32_t)c, v);
+      if (m < M) epi_chunk<bf16, 32>(e, m, n0, N, v);
+    }
+  } else if (!sw) {
+    // Staged epilogue: each 32-row x 32-column chunk is written into a
+    // swizzled shared-memory block and stored by one TMA copy (whole
+    // lines instead of one L2 request per 16 bytes).  The residual and
+    // history-base rows of a chunk are loaded ahead: the first chunk's
+    // before the accumulator wait, the next one's while the current
+    // chunk is finished.
+    const int m = t.m0 + row;
+    for (int c = c_lo; c < c_lo + BN / 2; c += 32) {
+      const int n0 = t.n0 + c;
+      if (n0 >= N) break;
+      float v[32];
+      tmem_ld32(tq + (uint32_t)c, v);
+      // y = gate * act(rope(acc + bias)), the order of epi_math; rows
+      // past M are not stored (the TMA store clips them)
+      if (e.bias) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, pb, j);
+      }
+      if (m < M) epi_rope_act<bf16, 32>(e, m, n0, v);
+      if (e.gate) {
+        const bool lo = m >= M || epi_batch(e, m) == b_lo;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const float g0 = __shfl_sync(0xffffffffu, pg0, j), g1 = __shfl_sync(0xffffffffu, pg1, j);
+          v[j] *= lo ? g0 : g1;
+        }
+      }
+      if (pre) {
+        if (!pre_ready()) { ok = 0; break; }
+        const uint8_t* rb = rsm + ((c - c_lo) >> 5) * 2048;
+        const uint8_t* hb2 = hsm + ((c - c_lo) >> 5) * 2048;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          if (pre & 1) pr[k] = *reinterpret_cast<const uint4*>(rb + blk_off(lane, k));
+          if (pre & 2) ph[k] = *reinterpret_cast<const uint4*>(hb2 + blk_off(lane, k));
+        }
+      }
+      uint32_t ob[16], hb[16];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t rr[4] = {pr[k].x, pr[k].y, pr[k].z, pr[k].w};
+        const uint32_t hh[4] = {ph[k].x, ph[k].y, ph[k].z, ph[k].w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          float a = v[8 * k + 2 * i], b = v[8 * k + 2 * i + 1];
+          if (e.resid) {
+            const float2 r2 = unpack2(rr[i]);
+            a += r2.x;
+            b += r2.y;
+          }
+          ob[4 * k + i] = pack2(a, b);
+          if (e.hist_out) {  // stored(out) - hist_base
+            const float2 o2 = unpack2(ob[4 * k + i]), h2 = unpack2(hh[i]);
+            hb[4 * k + i] = pack2(o2.x - h2.x, o2.y - h2.y);
+          }
+        }
+      }
+      if (c + 32 < c_lo + BN / 2 && n0 + 32 < N) fetch(n0 + 32);
+      // block(s) for this chunk: out alternates between the two when
+      // there is no history stream, else out -> block 0, hist -> block 1
+      uint8_t* b0 = ep + (e.hist_out ? 0 : (epi_cnt & 1) * 2048);
+      if (lane == 0) {
+        if (e.hist_out) bulk_wait_read<0>(); else bulk_wait_read<1>();
+      }
+      __syncwarp();
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        *reinterpret_cast<uint4*>(b0 + blk_off(lane, k)) = make_uint4(ob[4 * k], ob[4 * k + 1], ob[4 * k + 2], ob[4 * k + 3]);
+        if (e.hist_out)
+          *reinterpret_cast<uint4*>(ep + 2048 + blk_off(lane, k)) =
+              make_uint4(hb[4 * k], hb[4 * k + 1], hb[4 * k + 2], hb[4 * k + 3]);
+      }
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store(tmO, b0, n0, t.m0 + q * 32);
+        if (e.hist_out) tma_store(tmH, ep + 2048, n0, t.m0 + q * 32);
+        bulk_commit();
+      }
+      ++epi_cnt;
+    }
+  } else if constexpr (C::XPOSE_BYTES > 0) {
+    // lane = output column n + lane; TMEM column = output row.  Blocks of
+    // 16 rows x 32 columns go through the warp's buffer (XOR-swizzled,
+    // conflict-free both ways); afterwards lane l holds row l / 2,
+    // columns 16 (l % 2) .. + 15.
+    const int n = t.n0 + q * 32;
+    if (lane == 0) bulk_wait_read<0>();  // TMA stores of earlier tiles done reading the buffer
+    __syncwarp();
+    // preloaded form: the lane's 16 columns are the same for every block
+    // of rows, so their bias stays in registers and the gate row is
+    // reloaded only when the row's sample changes
+    const bool pre_sw = pre && !e.out_f32 && e.split_col >= N && !e.rope;
+    float bv[16], gv[16];
+    int gb = -1;
+    if (pre_sw) {
+      const int nc0 = n + (lane & 1) * 16;
+#pragma unroll
+      for (int g = 0; g < 2; ++g) {
+        float b8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (e.bias && nc0 + 8 * g < N) ld16(reinterpret_cast<const bf16*>(e.bias) + nc0 + 8 * g, b8);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) bv[8 * g + k] = b8[k];
+      }
+    }
+    for (int c = h * (BN / 2); c < (h + 1) * (BN / 2) && n < N; c += 16) {
+      const int m0 = t.m0 + c;
+      if (m0 >= M) break;
+      {
+        float u[16];
+        tmem_ld16(tq + (uint32_t)c, u);  // u[j] = out[m0 + j][n + lane]
+#pragma unroll
+        for (int j = 0; j < 16; ++j) xp[j * 32 + (lane ^ j)] = u[j];
+      }
+      __syncwarp();
+      const int r = lane >> 1, c0 = (lane & 1) * 16;
+      float v[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = xp[r * 32 + ((c0 + j) ^ r)];  // out[m0 + r][n + c0 + j]
+      __syncwarp();
+      const int m = m0 + r;
+      if (pre && !e.out_f32 && e.split_col >= N) {
+        // residual / history base of row m from the warp's ring slices
+        // (block (row in the warp's 128 rows) / 32, 16-byte chunks
+        // c0 / 8 and c0 / 8 + 1 of that row)
+        if (!pre_ready()) break;
+        if (m < M) {
+          if (pre_sw) {  // epi_math's order: act(acc + bias) * gate
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] += bv[j];
+            epi_rope_act<bf16, 16>(e, m, n + c0, v);
+            if (e.gate) {
+              const int bt = epi_batch(e, m);
+              if (bt != gb) {
+                gb = bt;
+                const float* gp = e.gate + (size_t)bt * e.gate_stride + n + c0;
+#pragma unroll
+                for (int j = 0; j < 16; j += 4) {
+                  const float4 g4 = n + c0 + j < N ? *reinterpret_cast<const float4*>(gp + j)
+                                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+                  gv[j] = g4.x; gv[j + 1] = g4.y; gv[j + 2] = g4.z; gv[j + 3] = g4.w;
+                }
+              }
+#pragma unroll
+              for (int j = 0; j < 16; ++j) v[j] *= gv[j];
+            }
+          } else {
+            epi_math<bf16, 16>(e, m, n + c0, N, v);
+          }
+          const int rw = c - h * (BN / 2) + r;
+          const uint32_t base = (uint32_t)((rw >> 5) * 2048);
+#pragma unroll
+          for (int g = 0; g < 2; ++g) {
+            const int nc = n + c0 + 8 * g;
+            if (nc >= N) continue;
+            const uint32_t off = base + blk_off(rw & 31, (c0 >> 3) + g);
+            uint4 rv = make_uint4(0, 0, 0, 0), hv = make_uint4(0, 0, 0, 0);
+            if (pre & 1)
+              rv = *reinterpret_cast<const uint4*>(rsm + off);
+            else if (e.resid)
+              rv = *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.resid) + (size_t)m * e.ld_resid + nc);
+            if (e.hist_out)
+              hv = (pre & 2) ? *reinterpret_cast<const uint4*>(hsm + off)
+                                : *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.hist_base) +
+                                                                  (size_t)m * e.ldo + nc);
+            const uint32_t rr4[4] = {rv.x, rv.y, rv.z, rv.w}, hh4[4] = {hv.x, hv.y, hv.z, hv.w};
+            uint32_t ob[4], hb[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              float a = v[8 * g + 2 * i], b = v[8 * g + 2 * i + 1];
+              if (e.resid) {
+                const float2 r2 = unpack2(rr4[i]);
+                a += r2.x;
+                b += r2.y;
+              }
+              ob[i] = pack2(a, b);
+              if (e.hist_out) {  // stored(out) - hist_base
+                const float2 o2 = unpack2(ob[i]), h2 = unpack2(hh4[i]);
+                hb[i] = pack2(o2.x - h2.x, o2.y - h2.y);
+              }
+            }
+            *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(e.out) + (size_t)m * e.ldo + nc) =
+                make_uint4(ob[0], ob[1], ob[2], ob[3]);
+            if (e.hist_out)
+              *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(e.hist_out) + (size_t)m * e.ldo + nc) =
+                  make_uint4(hb[0], hb[1], hb[2], hb[3]);
+          }
+        }
+        continue;
+      }
+      if (m < M) epi_chunk<bf16, 16>(e, m, n + c0, N, v);
+    }
+  }
+  // a warp whose columns all lie past N never read its blocks: their
+  // copies still land before it moves on
+  if (pre_wait) pre_ready();
+  return true;
+}
+
+// GROUPED: a second problem (group 1, tm1.n_tiles > 0) of the same N and K
 // with its own A, W, rows and epilogue (the text stream of a two-stream
-// block beside the image stream), its tiles first in the tile list; only
-// normal tiles, no residual preloads.  In each loop body `e`, `M` and `tm`
-// name the tile's group.
-template <int BN>
+// block beside the image stream), its tiles first in the tile list; both
+// groups then have only normal tiles and no residual preloads.  Without
+// GROUPED the group-1 parameters are unused.
+template <int BN, bool GROUPED>
 __global__ void __launch_bounds__(THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmW128, const __grid_constant__ CUtensorMap tmA256,
@@ -144,7 +445,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n1 = tm1.n_tiles;
+  const int n1 = GROUPED ? tm1.n_tiles : 0;
   const int num_tiles = tm0.n_tiles + n1;
   const int num_kb = (K + BK - 1) / BK;
 
@@ -164,7 +465,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
     if (tm0.pre & 1) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmR) : "memory");
     if (tm0.pre & 2) asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmHB) : "memory");
-    if (n1) {
+    if (GROUPED && n1) {
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA1) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB1) : "memory");
     }
@@ -193,7 +494,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
-        const bool g1 = tile < n1;
+        const bool g1 = GROUPED && tile < n1;
         const TileAt t = g1 ? tile_at<BN>(tm1, tile) : tile_at<BN>(tm0, tile - n1);
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
@@ -258,290 +559,24 @@ __global__ void __launch_bounds__(THREADS, 1)
     // may access), column half h of the tile
     const int q = warp & 3;
     const int h = (warp - 2) >> 2;
-    const int row = q * 32 + lane;
+    const EpiWarp W = {smem, reinterpret_cast<uint8_t*>(xpose) + (warp - 2) * 4096, rbar, tfull, abort_flag,
+                       tmem_base, warp, lane, q, h, q * 32 + lane, h * (BN / 2)};
     int tc = 0;
-    uint8_t* ep = reinterpret_cast<uint8_t*>(xpose) + (warp - 2) * 4096;
-    float* xp = reinterpret_cast<float*>(ep);
     uint32_t epi_cnt = 0;
-    const int c_lo = h * (BN / 2);
-    uint4 pr[4], ph[4];
-    float pb = 0.f, pg0 = 0.f, pg1 = 0.f;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++tc) {
-      const bool g1 = tile < n1;
-      const EpiArgs& e = g1 ? e1 : e0;
-      const TileMap& tm = g1 ? tm1 : tm0;
-      const int M = g1 ? M1 : M0;
-      const TileAt t = tile_at<BN>(tm, g1 ? tile : tile - n1);
       const int acc = tc & 1;
       const uint32_t aph = (tc >> 1) & 1;
-      // staged epilogue: residual / history-base rows of chunk n0 into pr /
-      // ph; bias and gate of column n0 + lane into pb / pg0 / pg1 (shared
-      // across the warp by shuffles: the warp's 32 rows lie in samples
-      // b_lo .. b_hi, at most two of them)
-      const int wr0 = t.m0 + q * 32;
-      const int b_lo = e.gate ? epi_batch(e, min(wr0, M - 1)) : 0;
-      const int b_hi = e.gate ? epi_batch(e, min(wr0 + 31, M - 1)) : 0;
-      auto fetch = [&](int n0) {
-        const int m = t.m0 + row;
-        const bool cin = n0 + lane < N;
-        pb = (e.bias && cin) ? __bfloat162float(reinterpret_cast<const bf16*>(e.bias)[n0 + lane]) : 0.f;
-        pg0 = (e.gate && cin) ? e.gate[(size_t)b_lo * e.gate_stride + n0 + lane] : 0.f;
-        pg1 = (e.gate && cin && b_hi != b_lo) ? e.gate[(size_t)b_hi * e.gate_stride + n0 + lane] : pg0;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const bool in = m < M && n0 + 8 * k < N;
-          if (e.resid && !(tm.pre & 1))
-            pr[k] = in ? *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.resid) +
-                                                          (size_t)m * e.ld_resid + n0 + 8 * k)
-                       : make_uint4(0, 0, 0, 0);
-          if (e.hist_out && !(tm.pre & 2))
-            ph[k] = in ? *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.hist_base) +
-                                                          (size_t)m * e.ldo + n0 + 8 * k)
-                       : make_uint4(0, 0, 0, 0);
-        }
-      };
-      if (C::XPOSE_BYTES > 0 && tm.staged && !t.sw) fetch(t.n0 + c_lo);
-      int ok = 1;
-      if (lane == 0) ok = mbar_wait_g(&tfull[acc], aph, abort_flag) ? 1 : 0;
-      ok = __shfl_sync(0xffffffffu, ok, 0);
+      bool ok;
+      if constexpr (GROUPED) {
+        ok = tile < n1 ? epi_tile<BN, true>(W, e1, tm1, M1, N, tile_at<BN>(tm1, tile), acc, aph, epi_cnt, &tmO1,
+                                            &tmH1, &tmR, &tmHB)
+                       : epi_tile<BN, true>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile - n1), acc, aph, epi_cnt, &tmO,
+                                            &tmH, &tmR, &tmHB);
+      } else {
+        ok = epi_tile<BN, false>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile), acc, aph, epi_cnt, &tmO, &tmH, &tmR,
+                                 &tmHB);
+      }
       if (!ok) break;
-      tc_fence_after();
-      // One tile per CTA: the ring's last readers (this tile's MMAs) are
-      // complete, so the warp's residual / history-base blocks (4 x 32 x 32
-      // bf16 each, 64-byte swizzle: the layout of the output blocks) come by
-      // TMA into its 8 KB slices of the ring; waited for at first use.
-      uint8_t* rsm = smem + (warp - 2) * 8192;
-      uint8_t* hsm = smem + 65536 + (warp - 2) * 8192;
-      bool pre_wait = tm.pre != 0;
-      if (tm.pre && lane == 0) {
-        mbar_expect_tx(&rbar[warp - 2], ((tm.pre & 1) ? 8192u : 0u) + ((tm.pre & 2) ? 8192u : 0u));
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int x = t.sw ? t.n0 + q * 32 : t.n0 + c_lo + 32 * i;
-          const int y = t.sw ? t.m0 + h * (BN / 2) + 32 * i : t.m0 + q * 32;
-          if (tm.pre & 1) tma_load(&tmR, &rbar[warp - 2], rsm + i * 2048, x, y);
-          if (tm.pre & 2) tma_load(&tmHB, &rbar[warp - 2], hsm + i * 2048, x, y);
-        }
-      }
-      auto pre_ready = [&]() -> bool {
-        if (!pre_wait) return true;
-        pre_wait = false;
-        int w = 1;
-        if (lane == 0) w = mbar_wait_g(&rbar[warp - 2], 0, abort_flag) ? 1 : 0;
-        return __shfl_sync(0xffffffffu, w, 0) != 0;
-      };
-      const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-      if (!t.sw && (C::XPOSE_BYTES == 0 || !tm.staged)) {
-        const int m = t.m0 + row;
-        for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
-          const int n0 = t.n0 + c;
-          if (n0 >= N) break;
-          float v[32];
-          tmem_ld32(tq + (uint32_t)c, v);
-          if (m < M) epi_chunk<bf16, 32>(e, m, n0, N, v);
-        }
-      } else if (!t.sw) {
-        // Staged epilogue: each 32-row x 32-column chunk is written into a
-        // swizzled shared-memory block and stored by one TMA copy (whole
-        // lines instead of one L2 request per 16 bytes).  The residual and
-        // history-base rows of a chunk are loaded ahead: the first chunk's
-        // before the accumulator wait, the next one's while the current
-        // chunk is finished.
-        const int m = t.m0 + row;
-        for (int c = c_lo; c < c_lo + BN / 2; c += 32) {
-          const int n0 = t.n0 + c;
-          if (n0 >= N) break;
-          float v[32];
-          tmem_ld32(tq + (uint32_t)c, v);
-          // y = gate * act(rope(acc + bias)), the order of epi_math; rows
-          // past M are not stored (the TMA store clips them)
-          if (e.bias) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, pb, j);
-          }
-          if (m < M) epi_rope_act<bf16, 32>(e, m, n0, v);
-          if (e.gate) {
-            const bool lo = m >= M || epi_batch(e, m) == b_lo;
-#pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const float g0 = __shfl_sync(0xffffffffu, pg0, j), g1 = __shfl_sync(0xffffffffu, pg1, j);
-              v[j] *= lo ? g0 : g1;
-            }
-          }
-          if (tm.pre) {
-            if (!pre_ready()) { ok = 0; break; }
-            const uint8_t* rb = rsm + ((c - c_lo) >> 5) * 2048;
-            const uint8_t* hb2 = hsm + ((c - c_lo) >> 5) * 2048;
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              if (tm.pre & 1) pr[k] = *reinterpret_cast<const uint4*>(rb + blk_off(lane, k));
-              if (tm.pre & 2) ph[k] = *reinterpret_cast<const uint4*>(hb2 + blk_off(lane, k));
-            }
-          }
-          uint32_t ob[16], hb[16];
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const uint32_t rr[4] = {pr[k].x, pr[k].y, pr[k].z, pr[k].w};
-            const uint32_t hh[4] = {ph[k].x, ph[k].y, ph[k].z, ph[k].w};
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              float a = v[8 * k + 2 * i], b = v[8 * k + 2 * i + 1];
-              if (e.resid) {
-                const float2 r2 = unpack2(rr[i]);
-                a += r2.x;
-                b += r2.y;
-              }
-              ob[4 * k + i] = pack2(a, b);
-              if (e.hist_out) {  // stored(out) - hist_base
-                const float2 o2 = unpack2(ob[4 * k + i]), h2 = unpack2(hh[i]);
-                hb[4 * k + i] = pack2(o2.x - h2.x, o2.y - h2.y);
-              }
-            }
-          }
-          if (c + 32 < c_lo + BN / 2 && n0 + 32 < N) fetch(n0 + 32);
-          // block(s) for this chunk: out alternates between the two when
-          // there is no history stream, else out -> block 0, hist -> block 1
-          uint8_t* b0 = ep + (e.hist_out ? 0 : (epi_cnt & 1) * 2048);
-          if (lane == 0) {
-            if (e.hist_out) bulk_wait_read<0>(); else bulk_wait_read<1>();
-          }
-          __syncwarp();
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            *reinterpret_cast<uint4*>(b0 + blk_off(lane, k)) = make_uint4(ob[4 * k], ob[4 * k + 1], ob[4 * k + 2], ob[4 * k + 3]);
-            if (e.hist_out)
-              *reinterpret_cast<uint4*>(ep + 2048 + blk_off(lane, k)) =
-                  make_uint4(hb[4 * k], hb[4 * k + 1], hb[4 * k + 2], hb[4 * k + 3]);
-          }
-          fence_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            if (g1) {
-              tma_store(&tmO1, b0, n0, t.m0 + q * 32);
-              if (e.hist_out) tma_store(&tmH1, ep + 2048, n0, t.m0 + q * 32);
-            } else {
-              tma_store(&tmO, b0, n0, t.m0 + q * 32);
-              if (e.hist_out) tma_store(&tmH, ep + 2048, n0, t.m0 + q * 32);
-            }
-            bulk_commit();
-          }
-          ++epi_cnt;
-        }
-      } else if constexpr (C::XPOSE_BYTES > 0) {
-        // lane = output column n + lane; TMEM column = output row.  Blocks of
-        // 16 rows x 32 columns go through the warp's buffer (XOR-swizzled,
-        // conflict-free both ways); afterwards lane l holds row l / 2,
-        // columns 16 (l % 2) .. + 15.
-        const int n = t.n0 + q * 32;
-        if (lane == 0) bulk_wait_read<0>();  // TMA stores of earlier tiles done reading the buffer
-        __syncwarp();
-        // preloaded form: the lane's 16 columns are the same for every block
-        // of rows, so their bias stays in registers and the gate row is
-        // reloaded only when the row's sample changes
-        const bool pre_sw = tm.pre && !e.out_f32 && e.split_col >= N && !e.rope;
-        float bv[16], gv[16];
-        int gb = -1;
-        if (pre_sw) {
-          const int nc0 = n + (lane & 1) * 16;
-#pragma unroll
-          for (int g = 0; g < 2; ++g) {
-            float b8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-            if (e.bias && nc0 + 8 * g < N) ld16(reinterpret_cast<const bf16*>(e.bias) + nc0 + 8 * g, b8);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) bv[8 * g + k] = b8[k];
-          }
-        }
-        for (int c = h * (BN / 2); c < (h + 1) * (BN / 2) && n < N; c += 16) {
-          const int m0 = t.m0 + c;
-          if (m0 >= M) break;
-          {
-            float u[16];
-            tmem_ld16(tq + (uint32_t)c, u);  // u[j] = out[m0 + j][n + lane]
-#pragma unroll
-            for (int j = 0; j < 16; ++j) xp[j * 32 + (lane ^ j)] = u[j];
-          }
-          __syncwarp();
-          const int r = lane >> 1, c0 = (lane & 1) * 16;
-          float v[16];
-#pragma unroll
-          for (int j = 0; j < 16; ++j) v[j] = xp[r * 32 + ((c0 + j) ^ r)];  // out[m0 + r][n + c0 + j]
-          __syncwarp();
-          const int m = m0 + r;
-          if (tm.pre && !e.out_f32 && e.split_col >= N) {
-            // residual / history base of row m from the warp's ring slices
-            // (block (row in the warp's 128 rows) / 32, 16-byte chunks
-            // c0 / 8 and c0 / 8 + 1 of that row)
-            if (!pre_ready()) break;
-            if (m < M) {
-              if (pre_sw) {  // epi_math's order: act(acc + bias) * gate
-#pragma unroll
-                for (int j = 0; j < 16; ++j) v[j] += bv[j];
-                epi_rope_act<bf16, 16>(e, m, n + c0, v);
-                if (e.gate) {
-                  const int bt = epi_batch(e, m);
-                  if (bt != gb) {
-                    gb = bt;
-                    const float* gp = e.gate + (size_t)bt * e.gate_stride + n + c0;
-#pragma unroll
-                    for (int j = 0; j < 16; j += 4) {
-                      const float4 g4 = n + c0 + j < N ? *reinterpret_cast<const float4*>(gp + j)
-                                                       : make_float4(0.f, 0.f, 0.f, 0.f);
-                      gv[j] = g4.x; gv[j + 1] = g4.y; gv[j + 2] = g4.z; gv[j + 3] = g4.w;
-                    }
-                  }
-#pragma unroll
-                  for (int j = 0; j < 16; ++j) v[j] *= gv[j];
-                }
-              } else {
-                epi_math<bf16, 16>(e, m, n + c0, N, v);
-              }
-              const int rw = c - h * (BN / 2) + r;
-              const uint32_t base = (uint32_t)((rw >> 5) * 2048);
-#pragma unroll
-              for (int g = 0; g < 2; ++g) {
-                const int nc = n + c0 + 8 * g;
-                if (nc >= N) continue;
-                const uint32_t off = base + blk_off(rw & 31, (c0 >> 3) + g);
-                uint4 rv = make_uint4(0, 0, 0, 0), hv = make_uint4(0, 0, 0, 0);
-                if (tm.pre & 1)
-                  rv = *reinterpret_cast<const uint4*>(rsm + off);
-                else if (e.resid)
-                  rv = *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.resid) + (size_t)m * e.ld_resid + nc);
-                if (e.hist_out)
-                  hv = (tm.pre & 2) ? *reinterpret_cast<const uint4*>(hsm + off)
-                                    : *reinterpret_cast<const uint4*>(reinterpret_cast<const bf16*>(e.hist_base) +
-                                                                      (size_t)m * e.ldo + nc);
-                const uint32_t rr4[4] = {rv.x, rv.y, rv.z, rv.w}, hh4[4] = {hv.x, hv.y, hv.z, hv.w};
-                uint32_t ob[4], hb[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                  float a = v[8 * g + 2 * i], b = v[8 * g + 2 * i + 1];
-                  if (e.resid) {
-                    const float2 r2 = unpack2(rr4[i]);
-                    a += r2.x;
-                    b += r2.y;
-                  }
-                  ob[i] = pack2(a, b);
-                  if (e.hist_out) {  // stored(out) - hist_base
-                    const float2 o2 = unpack2(ob[i]), h2 = unpack2(hh4[i]);
-                    hb[i] = pack2(o2.x - h2.x, o2.y - h2.y);
-                  }
-                }
-                *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(e.out) + (size_t)m * e.ldo + nc) =
-                    make_uint4(ob[0], ob[1], ob[2], ob[3]);
-                if (e.hist_out)
-                  *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(e.hist_out) + (size_t)m * e.ldo + nc) =
-                      make_uint4(hb[0], hb[1], hb[2], hb[3]);
-              }
-            }
-            continue;
-          }
-          if (m < M) epi_chunk<bf16, 16>(e, m, n + c0, N, v);
-        }
-      }
-      // a warp whose columns all lie past N never read its blocks: their
-      // copies still land before it moves on
-      if (pre_wait) pre_ready();
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
     }
@@ -756,8 +791,9 @@ bool init_driver() {
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
     if (g_sms <= 0) g_sms = 148;
-    cudaFuncSetAttribute(k_gemm_tc<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<128>::SMEM);
-    cudaFuncSetAttribute(k_gemm_tc<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
+    cudaFuncSetAttribute(k_gemm_tc<128, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<128>::SMEM);
+    cudaFuncSetAttribute(k_gemm_tc<256, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
+    cudaFuncSetAttribute(k_gemm_tc<256, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
     cudaFuncSetAttribute(k_gemm_tc2<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<128>::SMEM);
     cudaFuncSetAttribute(k_gemm_tc2<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<256>::SMEM);
   });
@@ -865,7 +901,7 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
     }
     const int grid = (int)(t256 < g_sms ? t256 : g_sms);
     const TileMap none = {};
-    launch_pdl(k_gemm_tc<256>, grid, THREADS, Cfg<256>::SMEM, s, ma, mb, mw128, ma256, mo, mh, mr, mhb, M, N, K, tm,
+    launch_pdl(k_gemm_tc<256, false>, grid, THREADS, Cfg<256>::SMEM, s, ma, mb, mw128, ma256, mo, mh, mr, mhb, M, N, K, tm,
                e, ma, mb, mo, mh, 0, none, e);
   } else {
     tm.n_full = (N + 127) / 128;
@@ -874,7 +910,7 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
     if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, 128)) return cudaErrorInvalidValue;
     const int grid = (int)(t128 < g_sms ? t128 : g_sms);
     const TileMap none = {};
-    launch_pdl(k_gemm_tc<128>, grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, ma, mb, M, N, K, tm, e, ma,
+    launch_pdl(k_gemm_tc<128, false>, grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, ma, mb, M, N, K, tm, e, ma,
                mb, ma, mb, 0, none, e);
   }
   return launched();
@@ -925,7 +961,7 @@ cudaError_t gemm_tc_grouped(int M0, const void* A0, const void* W0, const EpiArg
     return cudaErrorInvalidValue;
   const long long tiles = (long long)t0.n_tiles + t1.n_tiles;
   const int grid = (int)(tiles < g_sms ? tiles : g_sms);
-  launch_pdl(k_gemm_tc<256>, grid, THREADS, Cfg<256>::SMEM, s, a0, b0, a0, a0, o0, h0, a0, a0, M0, N, K, t0, e0, a1,
+  launch_pdl(k_gemm_tc<256, true>, grid, THREADS, Cfg<256>::SMEM, s, a0, b0, a0, a0, o0, h0, a0, a0, M0, N, K, t0, e0, a1,
              b1, o1, h1, M1, t1, e1);
   return launched();
 }
