@@ -267,6 +267,9 @@ inline cudaError_t launched() {
 cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int nt, long long n, cudaStream_t s);
 cudaError_t launch_diff(DType dt, const void* a, const void* b, void* out, long long n, cudaStream_t s);
 size_t verify_workspace_bytes(long long n);
+// Queries how many paid-check clusters are resident at once (the launched
+// grid); done on first use, or here ahead of any stream capture.
+void verify_prepare();
 // Partial forwarding at a site: out <- h_f on selected rows (rmask, per
 // token row) or columns (cmask), h_d elsewhere; row width C.
 struct FwdMix {

@@ -146,6 +146,8 @@ cudaError_t launch_diff(DType dt, const void* a, const void* b, void* out, long 
 constexpr int VERIFY_THREADS = 256;
 constexpr int VERIFY_CLUSTER = 8;
 
+// Upper bound of the grid (and so of the partials in the workspace): up to
+// four CTAs per SM, whole clusters.
 static int verify_grid(long long n) {
   long long nvec = n / 4 + 1;
   long long want = (nvec + VERIFY_THREADS - 1) / VERIFY_THREADS;
@@ -183,10 +185,9 @@ __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_
   float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
   const long long nvec = n / V;
   const long long stride = (long long)gridDim.x * blockDim.x;
-  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += stride) {
-    float a[V], f[V];
-    draft_vec<T, NT>(u, h, w, i, a);
-    ld16(hf + i * V, f);
+  // One vector of u, the history and h_f, accumulated, stored (Verify) and
+  // mixed (partial forwarding).
+  auto one = [&](long long i, float (&a)[V], const float (&f)[V]) {
 #pragma unroll
     for (int q = 0; q < V; ++q) {
       const float ad = round_to(a[q], (T*)nullptr);  // h_d as it would be forwarded
@@ -206,6 +207,25 @@ __global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_
       for (int q = 0; q < V; ++q) o[q] = (rmask ? rmask[r] : cmask[c0 + q]) ? f[q] : a[q];
       st16(mix + i * V, o);
     }
+  };
+  // Two vectors per thread and iteration, all their loads issued before
+  // either is used: the grid holds at most four CTAs per SM (the partials
+  // stay small), so each thread keeps twice the bytes in flight instead.
+  long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  for (; i + stride < nvec; i += 2 * stride) {
+    float a[V], f[V], a2[V], f2[V];
+    draft_vec<T, NT>(u, h, w, i, a);
+    draft_vec<T, NT>(u, h, w, i + stride, a2);
+    ld16(hf + i * V, f);
+    ld16(hf + (i + stride) * V, f2);
+    one(i, a, f);
+    one(i + stride, a2, f2);
+  }
+  if (i < nvec) {
+    float a[V], f[V];
+    draft_vec<T, NT>(u, h, w, i, a);
+    ld16(hf + i * V, f);
+    one(i, a, f);
   }
   if (blockIdx.x == 0 && threadIdx.x < n - nvec * V) {
     const long long i = nvec * V + threadIdx.x;
@@ -273,11 +293,50 @@ __global__ void k_verify_finish(const double* __restrict__ partials, int nparts,
   }
 }
 
+// The launched grid: verify_grid's bound, cut to the clusters that are
+// resident at once.  Clusters of 8 CTAs must fit in one GPC, so four CTAs
+// per SM on every SM are not all co-resident; a grid sized to them left a
+// second wave of a few clusters that ran alone (measured: the paid check at
+// 0.6 of the copy rate, with drafts of the same size at 1.0).
+template <class T, int NT>
+static int verify_launch_grid(long long n) {
+  static int resident = -1;  // clusters resident at once (per kernel instance)
+  if (resident < 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(VERIFY_CLUSTER * 64);
+    cfg.blockDim = dim3(VERIFY_THREADS);
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = VERIFY_CLUSTER;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int nc = 0;
+    if (cudaOccupancyMaxActiveClusters(&nc, k_verify<T, NT>, &cfg) != cudaSuccess || nc <= 0) {
+      cudaGetLastError();
+      nc = 0;  // unknown: keep the bound
+    }
+    resident = nc;
+  }
+  int grid = verify_grid(n);
+  if (resident > 0 && grid > resident * VERIFY_CLUSTER) grid = resident * VERIFY_CLUSTER;
+  return grid;
+}
+
+void verify_prepare() {
+  verify_launch_grid<float, 1>(1); verify_launch_grid<float, 2>(1);
+  verify_launch_grid<float, 3>(1); verify_launch_grid<float, 4>(1);
+  verify_launch_grid<bf16, 1>(1); verify_launch_grid<bf16, 2>(1);
+  verify_launch_grid<bf16, 3>(1); verify_launch_grid<bf16, 4>(1);
+}
+
 template <class T>
 static cudaError_t verify_t(void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
                            int write_draft, double* sums, void* ws, cudaStream_t s, const FwdMix* fm,
                            unsigned int* done_ctr) {
-  const int grid = verify_grid(n);
+  const int grid = nt == 1 ? verify_launch_grid<T, 1>(n) : nt == 2 ? verify_launch_grid<T, 2>(n)
+                 : nt == 3 ? verify_launch_grid<T, 3>(n) : verify_launch_grid<T, 4>(n);
   double* parts = reinterpret_cast<double*>(ws);
   T* up = reinterpret_cast<T*>(u);
   const T* fp = reinterpret_cast<const T*>(hf);

@@ -1035,6 +1035,7 @@ featfix_status schedule_buffers(featfix_ctx* ctx, int steps, int K, int mode, in
     ctx->max_logs = nlog;
   }
   // the partials, then the completion counter of the one-launch reduction
+  verify_prepare();  // host-side occupancy query, kept out of the graph capture
   const size_t need = (verify_workspace_bytes(ctx->E) + 255) / 256 * 256 + 256;
   if (need > ctx->vws_bytes) {
     free_ptr(&ctx->vws);
