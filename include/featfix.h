@@ -91,6 +91,21 @@ enum { FEATFIX_PLAN_EXACT = 0, FEATFIX_PLAN_DRAFT = 1, FEATFIX_PLAN_SITE = 2 };
  * set is the base policy's and Verify and FeatFix share their caches.
  * Drafted steps then run per block (no telescoping).                       */
 #define FEATFIX_FLAG_SITE_UPDATES_HISTORY 4u
+/* FUSED_LN fuses each adaLN LayerNorm-modulation of Eq. 1 that sits between
+ * two dense layers into them (bf16 models, C a multiple of 64): the GEMM
+ * that produces a block input (the embedding, the out-projection, fc2 /
+ * linear2 of the previous block at a full-refresh or vanilla step) also
+ * writes x (1 + scale) and per-row statistics of x, and the next layer
+ * computes
+ *   LN(x)(1 + scale)W^T + shift W^T
+ *     = rstd [x (1 + scale)] W^T - rstd mean (1 + scale) W^T + shift W^T
+ * with per-sample tables (1 + scale) W^T and shift W^T made once per
+ * trajectory.  Blocks whose input is a draft (sites) and the final layer
+ * keep the row kernel.  Same value up to rounding.  Off by default: the
+ * extra epilogue work of the two GEMMs costs more than the row kernel it
+ * removes (measured on GB300: DiT-XL/2 sampling 918 -> 677 steps/s,
+ * HunyuanVideo 34.7 -> 31.3).                                              */
+#define FEATFIX_FLAG_FUSED_LN 8u
 
 /*
  * Model shape (Eq. 1's block B_l and the surrounding sampler).

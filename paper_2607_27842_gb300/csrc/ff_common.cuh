@@ -93,6 +93,30 @@ struct EpiArgs {
   int rope_period;       // image tokens per sample
   int rope_cols;         // columns < rope_cols (q and k) are rotated
   int rope_hd;           // head width d (pairs (2j, 2j+1) within a head)
+  // adaLN LayerNorm of the next layer fused across two GEMMs (bf16 tensor-
+  // core path; rows map to samples as for the gate).  With
+  //   LN(x) (1 + s) + sh = rstd (x - mean) (1 + s) + sh
+  // the next layer's product with W splits into
+  //   rstd * [x (1 + s)] W^T - rstd * mean * [(1 + s) W^T] + sh W^T.
+  // Producer (ln_out non-null): the stored output row also goes out scaled,
+  // ln_out = stored(out) * (1 + ln_scale[b, n]) (row stride ldo), and every
+  // 32-column chunk of the stored row leaves (sum, sum of squared deviations
+  // from the chunk mean) in ln_stats[m * ln_slots + n / 32].
+  const float* ln_scale;
+  int ln_stride;
+  void* ln_out;
+  float2* ln_stats;
+  int ln_slots;
+  // Consumer (ln_in non-null): the A operand is such a scaled copy, and
+  //   acc <- rstd * acc - rstd * mean * ln_c[b, n] + ln_d[b, n]
+  // comes before the bias; mean and rstd (eps 1e-6) of row m combine its
+  // ln_slots chunk statistics over ln_cols columns; ln_c = (1 + s) W^T and
+  // ln_d = sh W^T per sample, rows of ln_cd_stride floats.
+  const float2* ln_in;
+  int ln_cols;
+  const float* ln_c;
+  const float* ln_d;
+  int ln_cd_stride;
 };
 
 static inline EpiArgs epi_plain(void* out, int ldo) {
@@ -140,9 +164,99 @@ __device__ __forceinline__ void epi_rope_act(const EpiArgs& e, int m, int n0, fl
 // are skipped (N % vector width == 0).
 // The part of the epilogue before the residual: y = gate * act(acc + bias),
 // with RoPE applied to q / k columns.
-template <class T, int CH>
-__device__ __forceinline__ void epi_math(const EpiArgs& e, int m, int n0, int N, float (&v)[CH]) {
+// (rstd, rstd * mean) of row m for the fused LayerNorm's consumer, from the
+// row's 32-column chunk statistics: mean = sum / C and
+//   M2 = sum_i M2_i + sum_i 32 mean_i^2 - C mean^2.
+__device__ __forceinline__ float2 ln_row(const EpiArgs& e, int m) {
+  const float4* p = reinterpret_cast<const float4*>(e.ln_in + (size_t)m * e.ln_slots);
+  float s1 = 0.f, s2 = 0.f, s3 = 0.f;
+  for (int k = 0; k < e.ln_slots / 2; ++k) {
+    const float4 q = __ldg(p + k);
+    s1 += q.x + q.z;
+    s2 += q.y + q.w;
+    s3 = fmaf(q.x, q.x, fmaf(q.z, q.z, s3));
+  }
+  if (e.ln_slots & 1) {
+    const float2 q = __ldg(e.ln_in + (size_t)m * e.ln_slots + e.ln_slots - 1);
+    s1 += q.x;
+    s2 += q.y;
+    s3 = fmaf(q.x, q.x, s3);
+  }
+  const float C = (float)e.ln_cols;
+  const float mean = s1 / C;
+  const float m2 = fmaxf(s2 + s3 * (1.0f / 32.0f) - C * mean * mean, 0.f);
+  const float rstd = rsqrtf(m2 / C + 1e-6f);
+  return make_float2(rstd, rstd * mean);
+}
+
+// Consumer correction of CH accumulator columns n0.. of row m (sample b):
+// v <- rstd * v - rstd * mean * ln_c + ln_d.
+template <int CH>
+__device__ __forceinline__ void ln_correct(const EpiArgs& e, int b, int n0, int N, float2 lnr, float (&v)[CH]) {
+  const float* cr = e.ln_c + (size_t)b * e.ln_cd_stride + n0;
+  const float* dr = e.ln_d + (size_t)b * e.ln_cd_stride + n0;
+#pragma unroll
+  for (int j = 0; j < CH; j += 4) {
+    if (n0 + j < N) {
+      const float4 c4 = __ldg(reinterpret_cast<const float4*>(cr + j));
+      const float4 d4 = __ldg(reinterpret_cast<const float4*>(dr + j));
+      v[j] = fmaf(lnr.x, v[j], fmaf(-lnr.y, c4.x, d4.x));
+      v[j + 1] = fmaf(lnr.x, v[j + 1], fmaf(-lnr.y, c4.y, d4.y));
+      v[j + 2] = fmaf(lnr.x, v[j + 2], fmaf(-lnr.y, c4.z, d4.z));
+      v[j + 3] = fmaf(lnr.x, v[j + 3], fmaf(-lnr.y, c4.w, d4.w));
+    }
+  }
+}
+
+// Producer side for CH stored values x of row m (sample b), columns n0..:
+// writes ln_out = x * (1 + ln_scale) and returns the chunk's (sum, sum of
+// squared deviations from its mean).
+template <int CH>
+__device__ __forceinline__ float2 ln_emit(const EpiArgs& e, int m, int b, int n0, const float (&x)[CH]) {
+  const float* sc = e.ln_scale + (size_t)b * e.ln_stride + n0;
+  bf16* o = reinterpret_cast<bf16*>(e.ln_out) + (size_t)m * e.ldo + n0;
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < CH; j += 8) {
+    const float4 a4 = __ldg(reinterpret_cast<const float4*>(sc + j));
+    const float4 b4 = __ldg(reinterpret_cast<const float4*>(sc + j + 4));
+    const float t[8] = {x[j] * (1.f + a4.x), x[j + 1] * (1.f + a4.y), x[j + 2] * (1.f + a4.z),
+                        x[j + 3] * (1.f + a4.w), x[j + 4] * (1.f + b4.x), x[j + 5] * (1.f + b4.y),
+                        x[j + 6] * (1.f + b4.z), x[j + 7] * (1.f + b4.w)};
+    st16(o + j, t);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) s += x[j + q];
+  }
+  const float mean = s * (1.0f / CH);
+  float m2 = 0.f;
+#pragma unroll
+  for (int j = 0; j < CH; ++j) {
+    const float d = x[j] - mean;
+    m2 = fmaf(d, d, m2);
+  }
+  return make_float2(s, m2);
+}
+
+// Two 16-column halves of a 32-column chunk held by lanes l and l ^ 1
+// (every lane of the warp calls this): the chunk's (sum, M2) on both lanes.
+__device__ __forceinline__ float2 ln_pair(float2 st) {
+  const float os = __shfl_xor_sync(0xffffffffu, st.x, 1);
+  const float om = __shfl_xor_sync(0xffffffffu, st.y, 1);
+  const float d = (st.x - os) * (1.0f / 16.0f);
+  return make_float2(st.x + os, st.y + om + d * d * 8.0f);
+}
+
+__device__ __forceinline__ void ln_put(const EpiArgs& e, int m, int n0, float2 st) {
+  e.ln_stats[(size_t)m * e.ln_slots + (n0 >> 5)] = st;
+}
+
+// LNM (compile time): which sides of the fused LayerNorm the caller's
+// kernel instance handles -- bit 0 consumer (ln_in), bit 1 producer (ln_out).
+template <class T, int CH, int LNM = 3>
+__device__ __forceinline__ void epi_math(const EpiArgs& e, int m, int n0, int N, float (&v)[CH],
+                                         float2 lnr = make_float2(1.f, 0.f)) {
   constexpr int V = VecN<T>::n;
+  if ((LNM & 1) && e.ln_in) ln_correct<CH>(e, epi_batch(e, m), n0, N, lnr, v);
   if (e.bias) {
     const T* b = reinterpret_cast<const T*>(e.bias);
 #pragma unroll
@@ -168,10 +282,13 @@ __device__ __forceinline__ void epi_math(const EpiArgs& e, int m, int n0, int N,
   }
 }
 
-template <class T, int CH>
-__device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N, float (&v)[CH]) {
+// Returns the chunk's (sum, M2) of the stored values when the output feeds a
+// fused LayerNorm (ln_out; bf16, chunks of 16 or 32 whole columns), else 0.
+template <class T, int CH, int LNM = 3>
+__device__ __forceinline__ float2 epi_chunk(const EpiArgs& e, int m, int n0, int N, float (&v)[CH],
+                                            float2 lnr = make_float2(1.f, 0.f)) {
   constexpr int V = VecN<T>::n;
-  epi_math<T, CH>(e, m, n0, N, v);
+  epi_math<T, CH, LNM>(e, m, n0, N, v, lnr);
   if (e.resid) {
     const T* rs = reinterpret_cast<const T*>(e.resid) + (size_t)m * e.ld_resid + n0;
 #pragma unroll
@@ -223,6 +340,15 @@ __device__ __forceinline__ void epi_chunk(const EpiArgs& e, int m, int n0, int N
       }
     }
   }
+  if constexpr (sizeof(T) == 2 && CH % 8 == 0 && (LNM & 2) != 0) {
+    if (e.ln_out && !e.out_f32 && n0 + CH <= N) {
+      float x[CH];
+#pragma unroll
+      for (int j = 0; j < CH; ++j) x[j] = round_to(v[j], (T*)nullptr);
+      return ln_emit<CH>(e, m, epi_batch(e, m), n0, x);
+    }
+  }
+  return make_float2(0.f, 0.f);
 }
 
 // ---------------------------------------------------------------------------
@@ -284,6 +410,9 @@ struct FwdMix {
 cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int nt, const void* hf, long long n,
                           int write_draft, double* sums, void* ws, cudaStream_t s,
                           const FwdMix* mix = nullptr, unsigned int* done_ctr = nullptr);
+// Operand rows of the fused-LayerNorm correction GEMMs (see k_ln_ab).
+cudaError_t launch_ln_ab(DType dt, const float* mod, long long mod_stride, int rows, int C, const int2* jobs,
+                         int njobs, void* out, long long job_stride, cudaStream_t s);
 cudaError_t launch_ln_mod(DType dt, const void* x, void* out, long long rows, int C, const float* shift,
                           const float* scale, int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s);
 // Sinusoidal features of S model times (device array) -> [S, 256] in dt.

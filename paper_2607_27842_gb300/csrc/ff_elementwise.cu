@@ -367,6 +367,41 @@ cudaError_t launch_verify(DType dt, void* u, const Hist4& h, const float* w, int
 }
 
 // ---------------------------------------------------------------------------
+// Operand rows of the fused-LayerNorm correction GEMMs: for job j (one
+// LayerNorm of one block and stream) and modulation row r,
+//   out[j][2r] = 1 + scale_r,  out[j][2r + 1] = shift_r
+// (columns jobs[j].x and jobs[j].y of the row), so one GEMM with the layer's
+// weight gives (1 + s) W^T and sh W^T interleaved.
+// ---------------------------------------------------------------------------
+template <class T>
+__global__ void __launch_bounds__(256) k_ln_ab(const float* __restrict__ mod, long long mod_stride, int C,
+                                               const int2* __restrict__ jobs, T* __restrict__ out,
+                                               long long job_stride) {
+  pdl_trigger();
+  pdl_wait();
+  const int r = blockIdx.x, j = blockIdx.y;
+  const int2 jc = jobs[j];
+  const float* sc = mod + (size_t)r * mod_stride + jc.x;
+  const float* sh = mod + (size_t)r * mod_stride + jc.y;
+  T* o = out + (size_t)j * job_stride + (size_t)2 * r * C;
+  for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    o[c] = from_f<T>(1.0f + sc[c]);
+    o[C + c] = from_f<T>(sh[c]);
+  }
+}
+
+cudaError_t launch_ln_ab(DType dt, const float* mod, long long mod_stride, int rows, int C, const int2* jobs,
+                         int njobs, void* out, long long job_stride, cudaStream_t s) {
+  if (rows <= 0 || njobs <= 0) return cudaSuccess;
+  const dim3 grid(rows, njobs);
+  if (dt == F32)
+    launch_pdl(k_ln_ab<float>, grid, dim3(256), 0, s, mod, mod_stride, C, jobs, (float*)out, job_stride);
+  else
+    launch_pdl(k_ln_ab<bf16>, grid, dim3(256), 0, s, mod, mod_stride, C, jobs, (bf16*)out, job_stride);
+  return launched();
+}
+
+// ---------------------------------------------------------------------------
 // adaLN branch input: LN(x) (no affine, eps 1e-6) * (1 + scale_b) + shift_b.
 // One warp per row, the row held in registers (NCH 16-byte vectors per
 // lane): one global read, exact two-pass mean / variance, one write.

@@ -32,6 +32,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 namespace ff {
@@ -131,7 +132,7 @@ struct EpiWarp {
 // field access of the inner loops into a generic load).  PLAIN: normal
 // tiles without residual preloads (the second problem of a grouped launch).
 // Returns false when the accumulator wait gave up.
-template <int BN, bool PLAIN>
+template <int BN, bool PLAIN, int LN>
 __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, const TileMap& tm, const int M,
                                          const int N, const TileAt t, const int acc, const uint32_t aph,
                                          uint32_t& epi_cnt, const CUtensorMap* tmO, const CUtensorMap* tmH,
@@ -146,6 +147,7 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
   volatile int* const abort_flag = W.abort_flag;
   const uint32_t tmem_base = W.tmem_base;
   const int pre = PLAIN ? 0 : tm.pre;
+  constexpr int LNM = LN == 1 ? 1 : LN == 2 ? 2 : 0;
   const bool sw = !PLAIN && t.sw;
   uint4 pr[4], ph[4];
   float pb = 0.f, pg0 = 0.f, pg1 = 0.f;
@@ -208,12 +210,16 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
   const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
   if (!sw && (C::XPOSE_BYTES == 0 || !tm.staged)) {
     const int m = t.m0 + row;
+    const float2 lnr = ((LN == 1 && e.ln_in) && m < M) ? ln_row(e, m) : make_float2(1.f, 0.f);
     for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
       const int n0 = t.n0 + c;
       if (n0 >= N) break;
       float v[32];
       tmem_ld32(tq + (uint32_t)c, v);
-      if (m < M) epi_chunk<bf16, 32>(e, m, n0, N, v);
+      if (m < M) {
+        const float2 st = epi_chunk<bf16, 32, LNM>(e, m, n0, N, v, lnr);
+        if ((LN == 2 && e.ln_out)) ln_put(e, m, n0, st);
+      }
     }
   } else if (!sw) {
     // Staged epilogue: each 32-row x 32-column chunk is written into a
@@ -223,6 +229,8 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
     // before the accumulator wait, the next one's while the current
     // chunk is finished.
     const int m = t.m0 + row;
+    const int bm = m < M ? epi_batch(e, m) : 0;   // the row's sample (fused LayerNorm)
+    const float2 lnr = ((LN == 1 && e.ln_in) && m < M) ? ln_row(e, m) : make_float2(1.f, 0.f);
     for (int c = c_lo; c < c_lo + BN / 2; c += 32) {
       const int n0 = t.n0 + c;
       if (n0 >= N) break;
@@ -230,6 +238,7 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
       tmem_ld32(tq + (uint32_t)c, v);
       // y = gate * act(rope(acc + bias)), the order of epi_math; rows
       // past M are not stored (the TMA store clips them)
+      if ((LN == 1 && e.ln_in) && m < M) ln_correct<32>(e, bm, n0, N, lnr, v);
       if (e.bias) {
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, pb, j);
@@ -272,6 +281,16 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
             hb[4 * k + i] = pack2(o2.x - h2.x, o2.y - h2.y);
           }
         }
+      }
+      if ((LN == 2 && e.ln_out) && m < M) {  // the next layer's scaled copy and chunk statistics
+        float x[32];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const float2 f = unpack2(ob[k]);
+          x[2 * k] = f.x;
+          x[2 * k + 1] = f.y;
+        }
+        ln_put(e, m, n0, ln_emit<32>(e, m, bm, n0, x));
       }
       if (c + 32 < c_lo + BN / 2 && n0 + 32 < N) fetch(n0 + 32);
       // block(s) for this chunk: out alternates between the two when
@@ -342,6 +361,7 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
         // (block (row in the warp's 128 rows) / 32, 16-byte chunks
         // c0 / 8 and c0 / 8 + 1 of that row)
         if (!pre_ready()) break;
+        float2 lst = make_float2(0.f, 0.f);   // fused LayerNorm: this lane's 16-column statistics
         if (m < M) {
           if (pre_sw) {  // epi_math's order: act(acc + bias) * gate
 #pragma unroll
@@ -363,10 +383,13 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
               for (int j = 0; j < 16; ++j) v[j] *= gv[j];
             }
           } else {
-            epi_math<bf16, 16>(e, m, n + c0, N, v);
+            epi_math<bf16, 16, LNM>(e, m, n + c0, N, v);
           }
           const int rw = c - h * (BN / 2) + r;
           const uint32_t base = (uint32_t)((rw >> 5) * 2048);
+          float xs[16];   // stored values of the lane's 16 columns
+#pragma unroll
+          for (int j = 0; j < 16; ++j) xs[j] = 0.f;
 #pragma unroll
           for (int g = 0; g < 2; ++g) {
             const int nc = n + c0 + 8 * g;
@@ -392,8 +415,11 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
                 b += r2.y;
               }
               ob[i] = pack2(a, b);
+              const float2 o2 = unpack2(ob[i]);
+              xs[8 * g + 2 * i] = o2.x;
+              xs[8 * g + 2 * i + 1] = o2.y;
               if (e.hist_out) {  // stored(out) - hist_base
-                const float2 o2 = unpack2(ob[i]), h2 = unpack2(hh4[i]);
+                const float2 h2 = unpack2(hh4[i]);
                 hb[i] = pack2(o2.x - h2.x, o2.y - h2.y);
               }
             }
@@ -403,10 +429,20 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
               *reinterpret_cast<uint4*>(reinterpret_cast<bf16*>(e.hist_out) + (size_t)m * e.ldo + nc) =
                   make_uint4(hb[0], hb[1], hb[2], hb[3]);
           }
+          if ((LN == 2 && e.ln_out)) lst = ln_emit<16>(e, m, epi_batch(e, m), n + c0, xs);
+        }
+        if ((LN == 2 && e.ln_out)) {  // lanes l and l ^ 1 hold the two halves of the row's 32 columns
+          lst = ln_pair(lst);
+          if (!(lane & 1) && m < M) ln_put(e, m, n, lst);
         }
         continue;
       }
-      if (m < M) epi_chunk<bf16, 16>(e, m, n + c0, N, v);
+      float2 lst = make_float2(0.f, 0.f);
+      if (m < M) lst = epi_chunk<bf16, 16, LNM>(e, m, n + c0, N, v, (LN == 1 && e.ln_in) ? ln_row(e, m) : make_float2(1.f, 0.f));
+      if ((LN == 2 && e.ln_out)) {
+        lst = ln_pair(lst);
+        if (!(lane & 1) && m < M) ln_put(e, m, n, lst);
+      }
     }
   }
   // a warp whose columns all lie past N never read its blocks: their
@@ -420,7 +456,7 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
 // block beside the image stream), its tiles first in the tile list; both
 // groups then have only normal tiles and no residual preloads.  Without
 // GROUPED the group-1 parameters are unused.
-template <int BN, bool GROUPED>
+template <int BN, bool GROUPED, int LN>
 __global__ void __launch_bounds__(THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmW128, const __grid_constant__ CUtensorMap tmA256,
@@ -568,12 +604,12 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t aph = (tc >> 1) & 1;
       bool ok;
       if constexpr (GROUPED) {
-        ok = tile < n1 ? epi_tile<BN, true>(W, e1, tm1, M1, N, tile_at<BN>(tm1, tile), acc, aph, epi_cnt, &tmO1,
+        ok = tile < n1 ? epi_tile<BN, true, LN>(W, e1, tm1, M1, N, tile_at<BN>(tm1, tile), acc, aph, epi_cnt, &tmO1,
                                             &tmH1, &tmR, &tmHB)
-                       : epi_tile<BN, true>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile - n1), acc, aph, epi_cnt, &tmO,
+                       : epi_tile<BN, true, LN>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile - n1), acc, aph, epi_cnt, &tmO,
                                             &tmH, &tmR, &tmHB);
       } else {
-        ok = epi_tile<BN, false>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile), acc, aph, epi_cnt, &tmO, &tmH, &tmR,
+        ok = epi_tile<BN, false, LN>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile), acc, aph, epi_cnt, &tmO, &tmH, &tmR,
                                  &tmHB);
       }
       if (!ok) break;
@@ -752,12 +788,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       if (!ok) break;
       tc_fence_after();
       const int m = mb * 2 * BM + row;
+      const float2 lnr = (e.ln_in && m < M) ? ln_row(e, m) : make_float2(1.f, 0.f);
       for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
         const int n0 = nb * BN + c;
         if (n0 >= N) break;
         float v[32];
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN + c), v);
-        if (m < M) epi_chunk<bf16, 32>(e, m, n0, N, v);
+        if (m < M) {
+          const float2 st = epi_chunk<bf16, 32>(e, m, n0, N, v, lnr);
+          if (e.ln_out) ln_put(e, m, n0, st);
+        }
       }
       tc_fence_before();
       mbar_arrive_cluster(map_to(&tempty[acc], 0));
@@ -776,6 +816,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
+// k_gemm_tc instance for a fused-LayerNorm side (0 none, 1 consumer, 2 producer)
+template <int BN, bool G>
+auto gemm_fn(int ln) -> decltype(&k_gemm_tc<BN, G, 0>) {
+  return ln == 1 ? k_gemm_tc<BN, G, 1> : ln == 2 ? k_gemm_tc<BN, G, 2> : k_gemm_tc<BN, G, 0>;
+}
+int ln_side(const EpiArgs& e) { return e.ln_in ? 1 : e.ln_out ? 2 : 0; }
+// a fused LayerNorm side: one side per launch, bf16 output of whole
+// 32-column chunks for the producer, 16-byte aligned rows everywhere
+bool ln_ok(const EpiArgs& e, int N) {
+  if (e.ln_in && e.ln_out) return false;
+  if (e.ln_out && (e.out_f32 || N % 32 != 0 || e.split_col < N || e.ldo % 8 != 0 || !e.ln_scale || !e.ln_stats ||
+                   e.ln_stride % 4 != 0 || ((uintptr_t)e.ln_scale & 15) || ((uintptr_t)e.ln_out & 15) ||
+                   e.ln_slots * 32 < N))
+    return false;
+  if (e.ln_in && (!e.ln_c || !e.ln_d || e.ln_cols <= 0 || e.ln_slots * 32 != e.ln_cols || (e.ln_slots & 1) ||
+                  e.ln_cd_stride % 4 != 0 ||
+                  ((uintptr_t)e.ln_c & 15) || ((uintptr_t)e.ln_d & 15) || ((uintptr_t)e.ln_in & 15)))
+    return false;
+  return true;
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_once;
 int g_sms = 0;
@@ -791,9 +852,11 @@ bool init_driver() {
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
     if (g_sms <= 0) g_sms = 148;
-    cudaFuncSetAttribute(k_gemm_tc<128, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<128>::SMEM);
-    cudaFuncSetAttribute(k_gemm_tc<256, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
-    cudaFuncSetAttribute(k_gemm_tc<256, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
+    for (int ln = 0; ln < 3; ++ln) {
+      cudaFuncSetAttribute(gemm_fn<128, false>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<128>::SMEM);
+      cudaFuncSetAttribute(gemm_fn<256, false>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
+      cudaFuncSetAttribute(gemm_fn<256, true>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
+    }
     cudaFuncSetAttribute(k_gemm_tc2<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<128>::SMEM);
     cudaFuncSetAttribute(k_gemm_tc2<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<256>::SMEM);
   });
@@ -848,6 +911,7 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (!init_driver()) return cudaErrorNotSupported;
   if (K % 8 != 0 || lda % 8 != 0 || ldw % 8 != 0 || N % 8 != 0) return cudaErrorInvalidValue;
+  if (!ln_ok(e, N)) return cudaErrorInvalidValue;
   if (((uintptr_t)A & 15) || ((uintptr_t)W & 15)) return cudaErrorInvalidValue;
   CUtensorMap ma, mb;
   // Long reductions: CTA pairs (256-row tiles, each CTA stages half of W);
@@ -901,7 +965,7 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
     }
     const int grid = (int)(t256 < g_sms ? t256 : g_sms);
     const TileMap none = {};
-    launch_pdl(k_gemm_tc<256, false>, grid, THREADS, Cfg<256>::SMEM, s, ma, mb, mw128, ma256, mo, mh, mr, mhb, M, N, K, tm,
+    launch_pdl(gemm_fn<256, false>(ln_side(e)), grid, THREADS, Cfg<256>::SMEM, s, ma, mb, mw128, ma256, mo, mh, mr, mhb, M, N, K, tm,
                e, ma, mb, mo, mh, 0, none, e);
   } else {
     tm.n_full = (N + 127) / 128;
@@ -910,7 +974,7 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
     if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, 128)) return cudaErrorInvalidValue;
     const int grid = (int)(t128 < g_sms ? t128 : g_sms);
     const TileMap none = {};
-    launch_pdl(k_gemm_tc<128, false>, grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, ma, mb, M, N, K, tm, e, ma,
+    launch_pdl(gemm_fn<128, false>(ln_side(e)), grid, THREADS, Cfg<128>::SMEM, s, ma, mb, ma, mb, ma, mb, ma, mb, M, N, K, tm, e, ma,
                mb, ma, mb, 0, none, e);
   }
   return launched();
@@ -945,6 +1009,8 @@ cudaError_t gemm_tc_grouped(int M0, const void* A0, const void* W0, const EpiArg
   if (M1 <= 0) return gemm_tc(M0, N, K, A0, lda, W0, ldw, e0, s);
   if (M0 <= 0) return gemm_tc(M1, N, K, A1, lda, W1, ldw, e1, s);
   if (!init_driver()) return cudaErrorNotSupported;
+  if (!ln_ok(e0, N) || !ln_ok(e1, N) || (ln_side(e0) && ln_side(e1) && ln_side(e0) != ln_side(e1)))
+    return cudaErrorInvalidValue;
   // CTA-pair reductions and column counts that need swapped tiles run as
   // two launches
   if ((M0 >= 2 * BM && K >= 8192) || N % 256 != 0) {
@@ -961,7 +1027,8 @@ cudaError_t gemm_tc_grouped(int M0, const void* A0, const void* W0, const EpiArg
     return cudaErrorInvalidValue;
   const long long tiles = (long long)t0.n_tiles + t1.n_tiles;
   const int grid = (int)(tiles < g_sms ? tiles : g_sms);
-  launch_pdl(k_gemm_tc<256, true>, grid, THREADS, Cfg<256>::SMEM, s, a0, b0, a0, a0, o0, h0, a0, a0, M0, N, K, t0, e0, a1,
+  const int ln = std::max(ln_side(e0), ln_side(e1));
+  launch_pdl(gemm_fn<256, true>(ln), grid, THREADS, Cfg<256>::SMEM, s, a0, b0, a0, a0, o0, h0, a0, a0, M0, N, K, t0, e0, a1,
              b1, o1, h1, M1, t1, e1);
   return launched();
 }

@@ -75,6 +75,25 @@ struct featfix_ctx {
   float* bmodtab = nullptr;         // [(n_need + 1) * Bm, Nblk]; the last row block is for featfix_debug_block
   float* fmodtab = nullptr;         // [steps * Bm, 2C]
   int mod_row_override = -1;
+  // adaLN LayerNorm fused across GEMMs (bf16): the GEMM producing a block
+  // input also writes its scaled copy (into xm) and 32-column statistics
+  // (lnst); the next layer's GEMM corrects its accumulator per row with the
+  // per-sample tables (1 + s) W^T and sh W^T (lncd).  One job per LayerNorm
+  // of a block and stream.
+  bool lnf = false;
+  float2* lnst = nullptr;           // [T, C / 32]
+  float* lncd = nullptr;            // per job: [(row blocks) * Bm][2][N]: c row, d row
+  void* lnab = nullptr;             // per job: [2 * (row blocks) * Bm][C] operand rows (1 + scale), shift
+  int2* d_lnjobs = nullptr;         // per job: columns of its scale and shift chunks in a modulation row
+  std::vector<int2> lnjobs;
+  std::vector<int> lnjob_n;         // per job: N of the layer after the LayerNorm
+  std::vector<const void*> lnjob_w; // per job: that layer's weight
+  std::vector<int> lnjob_at;        // (4 l + 2 s + k) -> job, -1 if none (s 0 image / only, 1 text; k 0 qkv, 1 fc1)
+  std::vector<long long> lncd_off;  // per job: offset (floats) of its table in lncd
+  long long lnab_job = 0;           // elements of one job's operand rows
+  int ln_rb = 0;                    // row blocks the tables hold
+  bool ln_src[2] = {false, false};  // xm rows of stream s hold the scaled copy for the next LayerNorm
+  bool ln_next = false;             // the block being run feeds the next block's first LayerNorm
   // logs
   double* dsums = nullptr;
   int max_logs = 0;
@@ -473,6 +492,44 @@ cudaError_t ln_mod(featfix_ctx* c, const void* x, void* out, long long rows, con
                        seg_split, rpb0, rpb1, c->st);
 }
 
+bool ln_fused(const featfix_ctx* c) { return !c->lncd_off.empty(); }
+
+// The layer after LayerNorm k (0 before qkv / linear1, 1 before fc1) of
+// block l, stream s (0 image / only, 1 text) reads the scaled copy in xm:
+// its epilogue corrects the accumulator with the row statistics at `stats`
+// and step i's per-sample tables.  Rows map to samples by
+// seg_split / rpb0 / rpb1 (as for a gate).
+void ln_consume(featfix_ctx* c, EpiArgs& e, int i, int l, int s, int k, const float2* stats, int seg_split, int rpb0,
+                int rpb1) {
+  const int j = c->lnjob_at[4 * l + 2 * s + k];
+  const int rb = c->mod_row_override >= 0 ? c->mod_row_override : c->need_row[i];
+  const int n = c->lnjob_n[j];
+  const float* base = c->lncd + c->lncd_off[j] + (size_t)rb * c->Bm * 2 * n;
+  e.ln_in = stats;
+  e.ln_slots = c->C / 32;
+  e.ln_cols = c->C;
+  e.ln_c = base;
+  e.ln_d = base + n;
+  e.ln_cd_stride = 2 * n;
+  e.seg_split = seg_split;
+  e.rpb0 = rpb0;
+  e.rpb1 = rpb1;
+}
+
+// This layer's output is the input of a LayerNorm with the scale chunk
+// `scale_chunk` of m: its epilogue also writes the scaled copy (ln_out, at
+// the GEMM's rows of xm) and the row statistics (stats).  The caller sets
+// the row-to-sample mapping (the gate's).
+void ln_produce(featfix_ctx* c, EpiArgs& e, const Mod& m, int scale_chunk, void* ln_out, float2* stats) {
+  e.ln_scale = m.chunk(scale_chunk, c->C);
+  e.ln_stride = m.stride;
+  e.ln_out = ln_out;
+  e.ln_stats = stats;
+  e.ln_slots = c->C / 32;
+}
+
+float2* ln_rows(featfix_ctx* c, long long row0) { return c->lnst + row0 * (c->C / 32); }
+
 // Exact DiT block B_l (Eq. 1): u -> out, optional history increment out - u.
 featfix_status block_dit(featfix_ctx* ctx, int i, int l, const void* u, void* out, void* hist) {
   const int C = ctx->C, M = ctx->M, es = ctx->es;
@@ -480,22 +537,35 @@ featfix_status block_dit(featfix_ctx* ctx, int i, int l, const void* u, void* ou
   const int wb = 11 + 10 * l;
   const auto& W = ctx->w;
   const Mod m = block_mod(ctx, i, l, 0);
-  FF_CK(ln_mod(ctx, u, ctx->xm, T, m, 0, 1, 0, 1, ctx->Ni));
-  FF_CK(dense(ctx, (int)T, 3 * C, C, ctx->xm, C, W[wb + 2], epi(ctx->qkv, 3 * C, W[wb + 3])));
+  const bool fz = ln_fused(ctx);
+  EpiArgs eq = epi(ctx->qkv, 3 * C, W[wb + 3]);
+  if (fz && ctx->ln_src[0])
+    ln_consume(ctx, eq, i, l, 0, 0, ctx->lnst, 0, 1, ctx->Ni);
+  else
+    FF_CK(ln_mod(ctx, u, ctx->xm, T, m, 0, 1, 0, 1, ctx->Ni));
+  ctx->ln_src[0] = false;
+  FF_CK(dense(ctx, (int)T, 3 * C, C, ctx->xm, C, W[wb + 2], eq));
   FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, es), off(ctx->qkv, 2 * C, es), 3 * C, ctx->att, C));
   EpiArgs e = epi(ctx->u1, C, W[wb + 5]);
   e.gate = m.chunk(2, C); e.gate_stride = m.stride; e.rpb1 = ctx->Ni;
   e.resid = u; e.ld_resid = C;
+  if (fz) ln_produce(ctx, e, m, 4, ctx->xm, ctx->lnst);
   FF_CK(dense(ctx, (int)T, C, C, ctx->att, C, W[wb + 4], e));
-  FF_CK(ln_mod(ctx, ctx->u1, ctx->xm, T, m, 3, 4, 0, 1, ctx->Ni));
   EpiArgs e1 = epi(ctx->big, M, W[wb + 7]);
   e1.act = 1;
+  if (fz)
+    ln_consume(ctx, e1, i, l, 0, 1, ctx->lnst, 0, 1, ctx->Ni);
+  else
+    FF_CK(ln_mod(ctx, ctx->u1, ctx->xm, T, m, 3, 4, 0, 1, ctx->Ni));
   FF_CK(dense(ctx, (int)T, M, C, ctx->xm, C, W[wb + 6], e1));
   EpiArgs e2 = epi(out, C, W[wb + 9]);
   e2.gate = m.chunk(5, C); e2.gate_stride = m.stride; e2.rpb1 = ctx->Ni;
   e2.resid = ctx->u1; e2.ld_resid = C;
   if (hist) { e2.hist_base = u; e2.hist_out = hist; }
+  const bool feed = fz && ctx->ln_next;
+  if (feed) ln_produce(ctx, e2, block_mod(ctx, i, l + 1, 0), 1, ctx->xm, ctx->lnst);
   FF_CK(dense(ctx, (int)T, C, M, ctx->big, M, W[wb + 8], e2));
+  ctx->ln_src[0] = feed;
   return FEATFIX_OK;
 }
 
@@ -509,19 +579,27 @@ featfix_status block_dual(featfix_ctx* ctx, int i, int l, const void* u, void* o
   const long long rt = (long long)ctx->Bm * ctx->Nt, ri = (long long)ctx->Bm * ctx->Ni;
   const Mod mi = block_mod(ctx, i, l, 0), mt = block_mod(ctx, i, l, 1);
   const int ti = (int)ri, tt = (int)rt;
-  // per-stream views: s = 0 text, 1 image
+  const bool fz = ln_fused(ctx);
+  // per-stream views: s = 0 text, 1 image (fused-LayerNorm job stream: 1 text, 0 image)
   auto rows0 = [&](int s_) { return s_ == 0 ? 0LL : rt; };
+  auto rpb = [&](int s_) { return s_ ? ctx->Ni : ctx->Nt; };
+  auto job_s = [&](int s_) { return s_ ? 0 : 1; };
+  bool fin[2];
   for (int s = 0; s < 2; ++s) {
     const long long rows = s == 0 ? rt : ri;
-    if (rows)
+    fin[s] = fz && ctx->ln_src[job_s(s)];
+    if (rows && !fin[s])
       FF_CK(ln_mod(ctx, coff(u, rows0(s) * C, es), off(ctx->xm, rows0(s) * C, es), rows, s ? mi : mt, 0, 1, 0, 1,
-                   s ? ctx->Ni : ctx->Nt));
+                   rpb(s)));
   }
+  ctx->ln_src[0] = ctx->ln_src[1] = false;
   EpiArgs qi = epi(off(ctx->qkv, rt * 3 * C, es), 3 * C, W[wb + 5]);
   if (ctx->rope) {
     qi.rope = ctx->rope; qi.rope_row0 = 0; qi.rope_period = ctx->Ni; qi.rope_cols = 2 * C; qi.rope_hd = ctx->hd;
   }
-  const EpiArgs qt = epi(ctx->qkv, 3 * C, W[wb + 7]);
+  EpiArgs qt = epi(ctx->qkv, 3 * C, W[wb + 7]);
+  if (fin[1]) ln_consume(ctx, qi, i, l, 0, 0, ln_rows(ctx, rt), 0, 1, ctx->Ni);
+  if (fin[0]) ln_consume(ctx, qt, i, l, 1, 0, ln_rows(ctx, 0), 0, 1, ctx->Nt);
   FF_CK(dense2(ctx, ti, off(ctx->xm, rt * C, es), W[wb + 4], qi, tt, ctx->xm, W[wb + 6], qt, 3 * C, C, C));
   FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, es), off(ctx->qkv, 2 * C, es), 3 * C, ctx->att, C));
   EpiArgs pe[2];
@@ -529,29 +607,42 @@ featfix_status block_dual(featfix_ctx* ctx, int i, int l, const void* u, void* o
     const Mod& m = s ? mi : mt;
     const int wp = s ? wb + 8 : wb + 10;
     pe[s] = epi(off(ctx->u1, rows0(s) * C, es), C, W[wp + 1]);
-    pe[s].gate = m.chunk(2, C); pe[s].gate_stride = m.stride; pe[s].rpb1 = s ? ctx->Ni : ctx->Nt;
+    pe[s].gate = m.chunk(2, C); pe[s].gate_stride = m.stride; pe[s].rpb1 = rpb(s);
     pe[s].resid = coff(u, rows0(s) * C, es); pe[s].ld_resid = C;
+    if (fz) ln_produce(ctx, pe[s], m, 4, off(ctx->xm, rows0(s) * C, es), ln_rows(ctx, rows0(s)));
   }
   FF_CK(dense2(ctx, ti, off(ctx->att, rt * C, es), W[wb + 8], pe[1], tt, ctx->att, W[wb + 10], pe[0], C, C, C));
-  for (int s = 0; s < 2; ++s) {
-    const long long rows = s == 0 ? rt : ri;
-    if (rows)
-      FF_CK(ln_mod(ctx, off(ctx->u1, rows0(s) * C, es), off(ctx->xm, rows0(s) * C, es), rows, s ? mi : mt, 3, 4, 0,
-                   1, s ? ctx->Ni : ctx->Nt));
+  if (!fz) {
+    for (int s = 0; s < 2; ++s) {
+      const long long rows = s == 0 ? rt : ri;
+      if (rows)
+        FF_CK(ln_mod(ctx, off(ctx->u1, rows0(s) * C, es), off(ctx->xm, rows0(s) * C, es), rows, s ? mi : mt, 3, 4, 0,
+                     1, rpb(s)));
+    }
   }
+  // the next block's first LayerNorm (a dual block: per stream; a single
+  // block: one modulation for both streams)
+  const bool feed = fz && ctx->ln_next;
+  const bool next_dual = l + 1 < ctx->d.n_dual;
   EpiArgs f1[2], f2[2];
   for (int s = 0; s < 2; ++s) {
     const Mod& m = s ? mi : mt;
     const int wf = s ? wb + 12 : wb + 16;
     f1[s] = epi(off(ctx->big, rows0(s) * M, es), M, W[wf + 1]);
     f1[s].act = 1;
+    if (fz) ln_consume(ctx, f1[s], i, l, job_s(s), 1, ln_rows(ctx, rows0(s)), 0, 1, rpb(s));
     f2[s] = epi(off(out, rows0(s) * C, es), C, W[wf + 3]);
-    f2[s].gate = m.chunk(5, C); f2[s].gate_stride = m.stride; f2[s].rpb1 = s ? ctx->Ni : ctx->Nt;
+    f2[s].gate = m.chunk(5, C); f2[s].gate_stride = m.stride; f2[s].rpb1 = rpb(s);
     f2[s].resid = off(ctx->u1, rows0(s) * C, es); f2[s].ld_resid = C;
     if (hist) { f2[s].hist_base = coff(u, rows0(s) * C, es); f2[s].hist_out = off(hist, rows0(s) * C, es); }
+    if (feed)
+      ln_produce(ctx, f2[s], block_mod(ctx, i, l + 1, next_dual ? job_s(s) : 0), 1, off(ctx->xm, rows0(s) * C, es),
+                 ln_rows(ctx, rows0(s)));
   }
   FF_CK(dense2(ctx, ti, off(ctx->xm, rt * C, es), W[wb + 12], f1[1], tt, ctx->xm, W[wb + 16], f1[0], M, C, C));
   FF_CK(dense2(ctx, ti, off(ctx->big, rt * M, es), W[wb + 14], f2[1], tt, ctx->big, W[wb + 18], f2[0], C, M, M));
+  ctx->ln_src[0] = feed && ri > 0;
+  ctx->ln_src[1] = feed && rt > 0;
   return FEATFIX_OK;
 }
 
@@ -565,7 +656,10 @@ featfix_status block_single(featfix_ctx* ctx, int i, int l, const void* u, void*
   const long long T = ctx->T, rt = (long long)ctx->Bm * ctx->Nt;
   const Mod m = block_mod(ctx, i, l, 0);
   const int rpb0 = ctx->Nt > 0 ? ctx->Nt : 1;
-  FF_CK(ln_mod(ctx, u, ctx->xm, T, m, 0, 1, (int)rt, rpb0, ctx->Ni));
+  const bool fz = ln_fused(ctx);
+  const bool fin = fz && ctx->ln_src[0] && (rt == 0 || ctx->ln_src[1]);
+  if (!fin) FF_CK(ln_mod(ctx, u, ctx->xm, T, m, 0, 1, (int)rt, rpb0, ctx->Ni));
+  ctx->ln_src[0] = ctx->ln_src[1] = false;
   EpiArgs e = epi(ctx->qkv, 3 * C, W[wb + 3]);
   e.split_col = 3 * C;
   e.out2 = off(ctx->big, C, ctx->es);
@@ -574,6 +668,7 @@ featfix_status block_single(featfix_ctx* ctx, int i, int l, const void* u, void*
   if (ctx->rope) {
     e.rope = ctx->rope; e.rope_row0 = (int)rt; e.rope_period = ctx->Ni; e.rope_cols = 2 * C; e.rope_hd = ctx->hd;
   }
+  if (fin) ln_consume(ctx, e, i, l, 0, 0, ctx->lnst, (int)rt, rpb0, ctx->Ni);
   FF_CK(dense(ctx, (int)T, 3 * C + M, C, ctx->xm, C, W[wb + 2], e));
   FF_CK(run_attention(ctx, ctx->qkv, off(ctx->qkv, C, ctx->es), off(ctx->qkv, 2 * C, ctx->es), 3 * C, ctx->big,
                       C + M));
@@ -582,7 +677,10 @@ featfix_status block_single(featfix_ctx* ctx, int i, int l, const void* u, void*
   e2.seg_split = (int)rt; e2.rpb0 = rpb0; e2.rpb1 = ctx->Ni;
   e2.resid = u; e2.ld_resid = C;
   if (hist) { e2.hist_base = u; e2.hist_out = hist; }
+  const bool feed = fz && ctx->ln_next;
+  if (feed) ln_produce(ctx, e2, block_mod(ctx, i, l + 1, 0), 1, ctx->xm, ctx->lnst);
   FF_CK(dense(ctx, (int)T, C, C + M, ctx->big, C + M, W[wb + 4], e2));
+  ctx->ln_src[0] = ctx->ln_src[1] = feed;
   return FEATFIX_OK;
 }
 
@@ -634,15 +732,35 @@ featfix_status compute_mods(featfix_ctx* ctx, const void* cond, int lo, int hi) 
     EpiArgs eb = epi(ctx->bmodtab + (size_t)rb0 * Bm * ctx->Nblk, (int)ctx->Nblk, ctx->bmod);
     eb.out_f32 = 1;
     FF_CK(dense(ctx, nneed * Bm, (int)ctx->Nblk, C, A, C, ctx->wmod, eb));
+    if (ln_fused(ctx)) {
+      // fused-LayerNorm tables of these row blocks: for every LayerNorm job,
+      // rows (1 + scale) and shift times the next layer's weight
+      const int nr = nneed * Bm;
+      {
+        KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
+        FF_CK(launch_ln_ab(ctx->dt, ctx->bmodtab + (size_t)rb0 * Bm * ctx->Nblk, ctx->Nblk, nr, C, ctx->d_lnjobs,
+                           (int)ctx->lnjobs.size(), ctx->lnab, ctx->lnab_job, ctx->st));
+      }
+      for (size_t j = 0; j < ctx->lnjobs.size(); ++j) {
+        const int n = ctx->lnjob_n[j];
+        EpiArgs ec = epi_plain(ctx->lncd + ctx->lncd_off[j] + (size_t)rb0 * Bm * 2 * n, n);
+        ec.out_f32 = 1;
+        FF_CK(dense(ctx, 2 * nr, n, C, off(ctx->lnab, (long long)j * ctx->lnab_job, es), C, ctx->lnjob_w[j], ec));
+      }
+    }
   }
   return FEATFIX_OK;
 }
 
 // Block-0 input: DiT patch embedding + position; MMDiT [text ; patches].
-featfix_status embed(featfix_ctx* ctx, const float* latent, const void* cond, void* x) {
+// feed: block 0 runs exact on this input, so the image rows' GEMM also
+// writes the scaled copy and statistics of block 0's first LayerNorm.
+featfix_status embed(featfix_ctx* ctx, int i, const float* latent, const void* cond, void* x, bool feed) {
   const auto& d = ctx->d;
   const int C = ctx->C, es = ctx->es;
   const long long rt = (long long)ctx->Bm * ctx->Nt;
+  feed = feed && ln_fused(ctx);
+  ctx->ln_src[0] = ctx->ln_src[1] = false;
   {
     KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
     FF_CK(launch_patchify(ctx->dt, latent, d.batch, ctx->Bm, d.in_ch, d.lat_f, d.lat_h, d.lat_w, d.patch, d.patch_t,
@@ -651,15 +769,20 @@ featfix_status embed(featfix_ctx* ctx, const float* latent, const void* cond, vo
   if (d.arch == FEATFIX_ARCH_DIT) {
     EpiArgs e = epi(x, C, ctx->w[6]);
     e.resid = ctx->pos; e.ld_resid = C;
+    e.rpb1 = ctx->Ni;
+    if (feed) ln_produce(ctx, e, block_mod(ctx, i, 0, 0), 1, ctx->xm, ctx->lnst);
     FF_CK(dense(ctx, ctx->Bm * ctx->Ni, C, ctx->fin, ctx->patches, ctx->fin, ctx->w[5], e));
   } else {
     if (rt) {
       KTimer tm(ctx, FEATFIX_KCLASS_OTHER, 0);
       FF_CK(launch_convert(ctx->dt, (const float*)cond, x, rt * C, ctx->st));
     }
-    FF_CK(dense(ctx, ctx->Bm * ctx->Ni, C, ctx->fin, ctx->patches, ctx->fin, ctx->w[4],
-                epi(off(x, rt * C, es), C, ctx->w[5])));
+    EpiArgs e = epi(off(x, rt * C, es), C, ctx->w[5]);
+    e.rpb1 = ctx->Ni;
+    if (feed) ln_produce(ctx, e, block_mod(ctx, i, 0, 0), 1, off(ctx->xm, rt * C, es), ln_rows(ctx, rt));
+    FF_CK(dense(ctx, ctx->Bm * ctx->Ni, C, ctx->fin, ctx->patches, ctx->fin, ctx->w[4], e));
   }
+  ctx->ln_src[0] = feed;
   return FEATFIX_OK;
 }
 
@@ -717,6 +840,7 @@ featfix_status verify_shadow(featfix_ctx* ctx, int i, int nt, const float* wf) {
   FF_CK(cudaMemcpyAsync(ctx->shadow, ctx->x0buf, bytes, cudaMemcpyDeviceToDevice, ctx->st));
   for (int l = 0; l <= last; ++l) {
     if (ctx->kinds[(size_t)i * L + l] == FEATFIX_PLAN_SITE) {
+      ctx->ln_src[0] = ctx->ln_src[1] = false;
       FF_TRY(exact_block(ctx, i, l, ctx->shadow, ctx->xa, nullptr));
       ctx->cnt.paid_checks++;
       const int slot = (int)ctx->log_sites.size();
@@ -747,7 +871,10 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
   const bool refresh = ctx->isref[i] != 0;
   const bool vanilla = ctx->mode == FEATFIX_MODE_VANILLA;
   const size_t bytes = (size_t)ctx->E * ctx->es;
-  FF_TRY(embed(ctx, latent, cond, ctx->x0buf));
+  // all blocks exact and chained (full refresh, vanilla): each block's
+  // output GEMM also prepares the next block's first LayerNorm
+  const bool chain = refresh || vanilla;
+  FF_TRY(embed(ctx, i, latent, cond, ctx->x0buf, chain && ctx->kinds[(size_t)i * L] == FEATFIX_PLAN_EXACT));
   const int new_slot = (ctx->head + 1) % ctx->S;
   const bool site_push = (ctx->flags & FEATFIX_FLAG_SITE_UPDATES_HISTORY) != 0;
   int nt = ctx->keff[i] + 1;
@@ -792,7 +919,9 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
       const int bslot = (ctx->bhead[l] + 1) % ctx->S;  // block l's next ring slot
       if (kind == FEATFIX_PLAN_EXACT) {
         void* hist = (refresh && !vanilla) ? ring_slot(ctx, l, bslot) : nullptr;
+        ctx->ln_next = chain && l + 1 < L;
         FF_TRY(exact_block(ctx, i, l, x, y, hist));
+        ctx->ln_next = false;
         advance();
       } else if (kind == FEATFIX_PLAN_DRAFT) {
         block_weights(l);
@@ -802,6 +931,7 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
         block_weights(l);
         // with site pushes the exact increment goes to the spare slot; the
         // draft below still reads the K_eff + 1 entries before it
+        ctx->ln_src[0] = ctx->ln_src[1] = false;  // the input comes from a draft
         FF_TRY(exact_block(ctx, i, l, x, y, site_push ? ring_slot(ctx, l, bslot) : nullptr));
         ctx->cnt.paid_checks++;
         if (ctx->mode != FEATFIX_MODE_EXACT_ONLY) {
@@ -886,7 +1016,7 @@ void free_all(featfix_ctx* c) {
   void* bufs[] = {c->xa, c->xb, c->xm, c->qkv, c->att, c->u1, c->big, c->patches, c->pos, c->mout, c->rope,
                   c->ring, c->sring, c->x0buf, c->shadow, c->wmod, c->bmod, c->d_times, c->d_need, c->sin_tab, c->thid_tab, c->temb_tab,
                   c->cs_all, c->cs_need, c->bmodtab, c->fmodtab, c->dsums, c->vws, c->g_lat, c->g_cond,
-                  c->h_latent, c->h_cond, c->d_rmask, c->d_cmask};
+                  c->h_latent, c->h_cond, c->d_rmask, c->d_cmask, c->lnst, c->lncd, c->lnab, c->d_lnjobs};
   for (void* p : bufs)
     if (p) cudaFree(p);
   for (int k = 0; k < NKCLASS; ++k)
@@ -977,6 +1107,45 @@ featfix_status gather_mod_weights(featfix_ctx* ctx) {
   return FEATFIX_OK;
 }
 
+// Jobs of the fused LayerNorm: every adaLN LayerNorm whose next layer is a
+// tensor-core GEMM -- DiT and dual blocks: before qkv (shift/scale chunks
+// 0/1) and before fc1 (3/4) per stream; single blocks: before linear1 (0/1).
+featfix_status setup_ln_jobs(featfix_ctx* ctx) {
+  const auto& d = ctx->d;
+  const long long C = ctx->C, M = ctx->M;
+  ctx->lnf = ctx->dt == BF16 && C % 64 == 0;   // an even number of 32-column chunks per row
+  ctx->lnjob_at.assign(4 * (size_t)ctx->L, -1);
+  if (!ctx->lnf) return FEATFIX_OK;
+  auto add = [&](int l, int s, int k, int w, long long n) {
+    const long long col = ctx->moff[2 * l + s];
+    const int shc = k == 0 ? 0 : 3, scc = k == 0 ? 1 : 4;
+    ctx->lnjob_at[4 * l + 2 * s + k] = (int)ctx->lnjobs.size();
+    ctx->lnjobs.push_back(make_int2((int)(col + scc * C), (int)(col + shc * C)));
+    ctx->lnjob_n.push_back((int)n);
+    ctx->lnjob_w.push_back(ctx->w[w]);
+  };
+  for (int l = 0; l < ctx->L; ++l) {
+    if (d.arch == FEATFIX_ARCH_DIT) {
+      const int wb = 11 + 10 * l;
+      add(l, 0, 0, wb + 2, 3 * C);
+      add(l, 0, 1, wb + 6, M);
+    } else if (l < d.n_dual) {
+      const int wb = 10 + 20 * l;
+      add(l, 0, 0, wb + 4, 3 * C);
+      add(l, 0, 1, wb + 12, M);
+      add(l, 1, 0, wb + 6, 3 * C);
+      add(l, 1, 1, wb + 16, M);
+    } else {
+      const int wb = 10 + 20 * d.n_dual + 6 * (l - d.n_dual);
+      add(l, 0, 0, wb + 2, 3 * C + M);
+    }
+  }
+  FF_TRY(alloc(ctx, (void**)&ctx->lnst, (size_t)ctx->T * (C / 32) * sizeof(float2)));
+  FF_TRY(alloc(ctx, (void**)&ctx->d_lnjobs, ctx->lnjobs.size() * sizeof(int2)));
+  FF_CK(cudaMemcpy(ctx->d_lnjobs, ctx->lnjobs.data(), ctx->lnjobs.size() * sizeof(int2), cudaMemcpyHostToDevice));
+  return FEATFIX_OK;
+}
+
 featfix_status create_impl(featfix_ctx* ctx) {
   const featfix_model_desc& d = ctx->d;
   const int es = ctx->es;
@@ -1009,6 +1178,7 @@ featfix_status create_impl(featfix_ctx* ctx) {
     FF_CK(cudaStreamSynchronize(ctx->user_st));
   }
   FF_TRY(gather_mod_weights(ctx));
+  FF_TRY(setup_ln_jobs(ctx));
   FF_CK(cudaStreamSynchronize(ctx->user_st));
   return FEATFIX_OK;
 }
@@ -1056,6 +1226,22 @@ featfix_status schedule_buffers(featfix_ctx* ctx, int steps, int K, int mode, in
   FF_TRY(alloc(ctx, &ctx->cs_need, (size_t)nn * Bm * C * es));
   FF_TRY(alloc(ctx, (void**)&ctx->bmodtab, (size_t)(nn + 1) * Bm * ctx->Nblk * 4));
   FF_TRY(alloc(ctx, (void**)&ctx->fmodtab, (size_t)steps * Bm * 2 * C * 4));
+  // fused-LayerNorm tables: one row block per modulation row block
+  free_ptr((void**)&ctx->lncd);
+  free_ptr(&ctx->lnab);
+  ctx->lncd_off.clear();
+  if (ctx->lnf && (flags & FEATFIX_FLAG_FUSED_LN)) {
+    const long long rows = (long long)(nn + 1) * Bm;
+    long long tot = 0;
+    for (int n : ctx->lnjob_n) {
+      ctx->lncd_off.push_back(tot);
+      tot += 2 * rows * n;
+    }
+    ctx->ln_rb = nn + 1;
+    ctx->lnab_job = 2 * rows * C;
+    FF_TRY(alloc(ctx, (void**)&ctx->lncd, (size_t)tot * 4));
+    FF_TRY(alloc(ctx, &ctx->lnab, (size_t)ctx->lnjobs.size() * ctx->lnab_job * es));
+  }
   return FEATFIX_OK;
 }
 
@@ -1392,6 +1578,8 @@ featfix_status featfix_debug_block(featfix_ctx* ctx, int step, int layer, const 
   ctx->need_row[step] = saved;
   if (s != FEATFIX_OK) return s;
   ctx->mod_row_override = spare;
+  ctx->ln_src[0] = ctx->ln_src[1] = false;
+  ctx->ln_next = false;
   s = exact_block(ctx, step, layer, dev_in, dev_out, nullptr);
   ctx->mod_row_override = -1;
   return s;

@@ -23,6 +23,7 @@ PLAN_EXACT, PLAN_DRAFT, PLAN_SITE = 0, 1, 2
 FLAG_TAYLOR_RECURSIVE = 1
 FLAG_PER_BLOCK_DRAFT = 2
 FLAG_SITE_UPDATES_HISTORY = 4
+FLAG_FUSED_LN = 8
 MASK_NONE, MASK_TOKENS, MASK_CHANNELS = 0, 1, 2
 KCLASS = {"gemm": 0, "attention": 1, "draft": 2, "verify": 3, "other": 4}
 

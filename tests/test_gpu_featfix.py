@@ -240,6 +240,28 @@ def test_telescoped_steps_match_per_block(case):
     assert rel_l2(a, b) < (1e-5 if case.sh.dtype == "f32" else 1e-2)
 
 
+def test_fused_layernorm_matches_standalone(case):
+    """Eq. 1's adaLN LayerNorm fused across the dense layers (FLAG_FUSED_LN,
+    bf16: the producing GEMM writes x(1 + scale) and row statistics, the
+    consuming GEMM corrects per row with (1 + scale)W^T and shift W^T) equals
+    the standalone row kernel up to rounding; fp32 never fuses."""
+    case.schedule("vanilla")
+    a = case.sample(seed=11).cpu().numpy()
+    case.schedule("vanilla", flags=ff.FLAG_FUSED_LN)
+    b = case.sample(seed=11).cpu().numpy()
+    if case.sh.dtype == "f32":
+        np.testing.assert_array_equal(a, b)
+    else:
+        assert 0 < rel_l2(a, b) < 1e-2
+    case.schedule("featfix")
+    a = case.sample(seed=11).cpu().numpy()
+    case.schedule("featfix", flags=ff.FLAG_FUSED_LN)
+    b = case.sample(seed=11).cpu().numpy()
+    assert rel_l2(a, b) < (1e-7 if case.sh.dtype == "f32" else 1e-2)
+    x_ref, _, _ = case.oracle_run("featfix", seed=11)
+    assert rel_l2(b, x_ref) < tol_latent(case.sh)
+
+
 def test_call_order_errors(cuda):
     c = Case(syn.workload("tiny"))
     try:
