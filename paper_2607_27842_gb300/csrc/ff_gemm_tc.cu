@@ -130,14 +130,14 @@ struct EpiWarp {
 // every EpiArgs / TileMap field and tensor map is read from its own kernel
 // parameter (a run-time choice between two parameter structs turns every
 // field access of the inner loops into a generic load).  PLAIN: normal
-// tiles without residual preloads (the second problem of a grouped launch).
-// Returns false when the accumulator wait gave up.
-template <int BN, bool PLAIN, int LN>
+// tiles without residual preloads (the second problem of a grouped launch,
+// the CTA pairs).  XB: bytes of the epilogue warps' staging buffers (0: the
+// per-lane store path only).  Returns false when the accumulator wait gave up.
+template <int BN, int XB, bool PLAIN, int LN>
 __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, const TileMap& tm, const int M,
                                          const int N, const TileAt t, const int acc, const uint32_t aph,
                                          uint32_t& epi_cnt, const CUtensorMap* tmO, const CUtensorMap* tmH,
                                          const CUtensorMap* tmR, const CUtensorMap* tmHB) {
-  using C = Cfg<BN>;
   const int warp = W.warp, lane = W.lane, q = W.q, h = W.h, row = W.row, c_lo = W.c_lo;
   uint8_t* const smem = W.smem;
   uint8_t* const ep = W.ep;
@@ -177,7 +177,7 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
                    : make_uint4(0, 0, 0, 0);
     }
   };
-  if (C::XPOSE_BYTES > 0 && tm.staged && !sw) fetch(t.n0 + c_lo);
+  if (XB > 0 && tm.staged && !sw) fetch(t.n0 + c_lo);
   int ok = 1;
   if (lane == 0) ok = mbar_wait_g(&tfull[acc], aph, abort_flag) ? 1 : 0;
   ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -208,7 +208,7 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
     return __shfl_sync(0xffffffffu, w, 0) != 0;
   };
   const uint32_t tq = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-  if (!sw && (C::XPOSE_BYTES == 0 || !tm.staged)) {
+  if (!sw && (XB == 0 || !tm.staged)) {
     const int m = t.m0 + row;
     const float2 lnr = ((LN == 1 && e.ln_in) && m < M) ? ln_row(e, m) : make_float2(1.f, 0.f);
     for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
@@ -316,7 +316,7 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
       }
       ++epi_cnt;
     }
-  } else if constexpr (C::XPOSE_BYTES > 0) {
+  } else if constexpr (XB > 0) {
     // lane = output column n + lane; TMEM column = output row.  Blocks of
     // 16 rows x 32 columns go through the warp's buffer (XOR-swizzled,
     // conflict-free both ways); afterwards lane l holds row l / 2,
@@ -604,12 +604,12 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t aph = (tc >> 1) & 1;
       bool ok;
       if constexpr (GROUPED) {
-        ok = tile < n1 ? epi_tile<BN, true, LN>(W, e1, tm1, M1, N, tile_at<BN>(tm1, tile), acc, aph, epi_cnt, &tmO1,
+        ok = tile < n1 ? epi_tile<BN, Cfg<BN>::XPOSE_BYTES, true, LN>(W, e1, tm1, M1, N, tile_at<BN>(tm1, tile), acc, aph, epi_cnt, &tmO1,
                                             &tmH1, &tmR, &tmHB)
-                       : epi_tile<BN, true, LN>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile - n1), acc, aph, epi_cnt, &tmO,
+                       : epi_tile<BN, Cfg<BN>::XPOSE_BYTES, true, LN>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile - n1), acc, aph, epi_cnt, &tmO,
                                             &tmH, &tmR, &tmHB);
       } else {
-        ok = epi_tile<BN, false, LN>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile), acc, aph, epi_cnt, &tmO, &tmH, &tmR,
+        ok = epi_tile<BN, Cfg<BN>::XPOSE_BYTES, false, LN>(W, e0, tm0, M0, N, tile_at<BN>(tm0, tile), acc, aph, epi_cnt, &tmO, &tmH, &tmR,
                                  &tmHB);
       }
       if (!ok) break;
@@ -644,38 +644,26 @@ template <int BN> struct Cfg2 {
   static constexpr uint32_t B_BYTES = HB * BK * 2;
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + 256;
+  static constexpr uint32_t XPOSE_BYTES = 8 * 4096;  // the staged epilogue's output blocks
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + XPOSE_BYTES + 256;
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                                     ((uint32_t)(256 >> 4) << 24);
 };
 
-__device__ __forceinline__ void umma_pair(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
-          d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(accum));
-}
-// arrive on the mbarrier at this offset in both CTAs of the pair once the
-// issued MMAs complete
-__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
-  const uint16_t mask = 3;
-  asm volatile(
-      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-          saddr(bar)),
-      "h"(mask)
-      : "memory");
-}
-
-template <int BN>
+// The epilogue is epi_tile's (staged TMA-store blocks where tm.staged), each
+// CTA on its own 128 rows of the pair's 256-row tile.
+template <int BN, int LN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
-    k_gemm_tc2(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
-               EpiArgs e) {
+    k_gemm_tc2(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmH, int M, int N, int K,
+               const __grid_constant__ TileMap tm, const __grid_constant__ EpiArgs e) {
   using C = Cfg2<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
+  uint8_t* xpose = sB + C::STAGES * C::B_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(xpose + C::XPOSE_BYTES);
   uint64_t* empty = full + C::STAGES;
   uint64_t* tfull = empty + C::STAGES;
   uint64_t* tempty = tfull + 2;
@@ -776,32 +764,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   } else {
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int h = (warp - 2) >> 2;  // column half of the tile
-    const int row = (int)rank * BM + q * 32 + lane;
+    const EpiWarp W = {smem, xpose + (warp - 2) * 4096, tfull, tfull, abort_flag, tmem_base, warp, lane, q, h,
+                       q * 32 + lane, h * (BN / 2)};
     int tc = 0;
+    uint32_t epi_cnt = 0;
     for (int tile = pair; tile < num_tiles; tile += npairs, ++tc) {
       const int mb = tile % num_m, nb = tile / num_m;
       const int acc = tc & 1;
       const uint32_t aph = (tc >> 1) & 1;
-      int ok = 1;
-      if (lane == 0) ok = mbar_wait_g(&tfull[acc], aph, abort_flag) ? 1 : 0;
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) break;
-      tc_fence_after();
-      const int m = mb * 2 * BM + row;
-      const float2 lnr = (e.ln_in && m < M) ? ln_row(e, m) : make_float2(1.f, 0.f);
-      for (int c = h * (BN / 2); c < (h + 1) * (BN / 2); c += 32) {
-        const int n0 = nb * BN + c;
-        if (n0 >= N) break;
-        float v[32];
-        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN + c), v);
-        if (m < M) {
-          const float2 st = epi_chunk<bf16, 32>(e, m, n0, N, v, lnr);
-          if (e.ln_out) ln_put(e, m, n0, st);
-        }
-      }
+      const TileAt t = {false, mb * 2 * BM + (int)rank * BM, nb * BN};
+      if (!epi_tile<BN, C::XPOSE_BYTES, true, LN>(W, e, tm, M, N, t, acc, aph, epi_cnt, &tmO, &tmH, &tmO, &tmO))
+        break;
       tc_fence_before();
       mbar_arrive_cluster(map_to(&tempty[acc], 0));
     }
+    if (lane == 0) bulk_wait_all();  // TMA stores complete before exit
   }
   tc_fence_before();
   __syncwarp();
@@ -820,6 +797,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 template <int BN, bool G>
 auto gemm_fn(int ln) -> decltype(&k_gemm_tc<BN, G, 0>) {
   return ln == 1 ? k_gemm_tc<BN, G, 1> : ln == 2 ? k_gemm_tc<BN, G, 2> : k_gemm_tc<BN, G, 0>;
+}
+template <int BN>
+auto gemm2_fn(int ln) -> decltype(&k_gemm_tc2<BN, 0>) {
+  return ln == 1 ? k_gemm_tc2<BN, 1> : ln == 2 ? k_gemm_tc2<BN, 2> : k_gemm_tc2<BN, 0>;
 }
 int ln_side(const EpiArgs& e) { return e.ln_in ? 1 : e.ln_out ? 2 : 0; }
 // a fused LayerNorm side: one side per launch, bf16 output of whole
@@ -857,8 +838,10 @@ bool init_driver() {
       cudaFuncSetAttribute(gemm_fn<256, false>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
       cudaFuncSetAttribute(gemm_fn<256, true>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<256>::SMEM);
     }
-    cudaFuncSetAttribute(k_gemm_tc2<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<128>::SMEM);
-    cudaFuncSetAttribute(k_gemm_tc2<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<256>::SMEM);
+    for (int ln = 0; ln < 3; ++ln) {
+      cudaFuncSetAttribute(gemm2_fn<128>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<128>::SMEM);
+      cudaFuncSetAttribute(gemm2_fn<256>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<256>::SMEM);
+    }
   });
   return g_encode != nullptr;
 }
@@ -889,6 +872,18 @@ bool make_store_map(CUtensorMap* m, void* base, int rows, int cols, int ld) {
   return r == CUDA_SUCCESS;
 }
 
+// The staged (TMA-store) epilogue: one bf16 output of 16-byte aligned rows,
+// plus the history stream when present, and a warp's 32 rows spanning at
+// most two gate rows.  Encodes the store maps; false where the per-lane
+// store path has to be used.
+bool staged_maps(const EpiArgs& e, int M, int N, CUtensorMap* mo, CUtensorMap* mh) {
+  const bool aligned = !((uintptr_t)e.out & 15) && e.ldo % 8 == 0 &&
+                       (!e.hist_out || (!((uintptr_t)e.hist_out & 15) && !((uintptr_t)e.hist_base & 15)));
+  const bool gate_ok = !e.gate || ((e.seg_split <= 0 || e.rpb0 >= 32) && e.rpb1 >= 32);
+  return !e.out_f32 && e.split_col >= N && aligned && gate_ok && make_store_map(mo, e.out, M, N, e.ldo) &&
+         (!e.hist_out || make_store_map(mh, e.hist_out, M, N, e.ldo));
+}
+
 // Tile width choice: the fewest waves of rows_per_tile x BN tiles over the
 // available CTAs (or CTA pairs), ties to the wider tile (less shared-memory
 // traffic per FLOP).
@@ -915,17 +910,23 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
   if (((uintptr_t)A & 15) || ((uintptr_t)W & 15)) return cudaErrorInvalidValue;
   CUtensorMap ma, mb;
   // Long reductions: CTA pairs (256-row tiles, each CTA stages half of W);
-  // measured faster than single CTAs only from K of about 8k on.
+  // measured faster than single CTAs only from K of about 8k on.  (256 x 128
+  // pair tiles for the one-wave DiT-XL/2 layers, two tiles per pair so that
+  // an epilogue runs beside the next mainloop, measured slower: fc2 44.8 ->
+  // 49.8 us, out-projection 19.1 -> 18.0 us.)
   if (M >= 2 * BM && K >= 8192) {
     const int pairs = g_sms / 2;
     const int bn = pick_bn(M, N, 2 * BM, pairs);
     if (!make_map(&ma, A, M, K, lda, BM) || !make_map(&mb, W, N, K, ldw, bn / 2)) return cudaErrorInvalidValue;
     const long long tiles = (long long)((M + 2 * BM - 1) / (2 * BM)) * ((N + bn - 1) / bn);
     const int grid = 2 * (int)(tiles < pairs ? tiles : pairs);
+    TileMap tm2 = {};
+    CUtensorMap mo = ma, mh = ma;
+    tm2.staged = staged_maps(e, M, N, &mo, &mh) ? 1 : 0;
     if (bn == 256)
-      launch_pdl(k_gemm_tc2<256>, grid, THREADS, Cfg2<256>::SMEM, s, ma, mb, M, N, K, e);
+      launch_pdl(gemm2_fn<256>(ln_side(e)), grid, THREADS, Cfg2<256>::SMEM, s, ma, mb, mo, mh, M, N, K, tm2, e);
     else
-      launch_pdl(k_gemm_tc2<128>, grid, THREADS, Cfg2<128>::SMEM, s, ma, mb, M, N, K, e);
+      launch_pdl(gemm2_fn<128>(ln_side(e)), grid, THREADS, Cfg2<128>::SMEM, s, ma, mb, mo, mh, M, N, K, tm2, e);
     return launched();
   }
   // Every tile (128 x 256 full rate, 128 x 128 at half rate, swapped 128 x

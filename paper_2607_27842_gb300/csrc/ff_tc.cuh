@@ -125,6 +125,25 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 
+// CTA-pair MMA (M = 256: each CTA's 128 rows of A and accumulator, each CTA
+// half of B along N), both operands from shared memory
+__device__ __forceinline__ void umma_pair(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+          d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accum));
+}
+// arrive on the mbarrier at this offset in both CTAs of the pair once the
+// issued MMAs complete
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
+  const uint16_t mask = 3;
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          saddr(bar)),
+      "h"(mask)
+      : "memory");
+}
+
 // Shared-memory matrix descriptor, K-major operand with 128-byte swizzle:
 // start address >> 4 (bits 0-13), leading offset 1 (unused for swizzled
 // K-major), stride offset 1024 B between 8-row groups (bits 32-45),
