@@ -245,11 +245,16 @@ __device__ __forceinline__ bool epi_tile(const EpiWarp& W, const EpiArgs& e, con
       }
       if (m < M) epi_rope_act<bf16, 32>(e, m, n0, v);
       if (e.gate) {
-        const bool lo = m >= M || epi_batch(e, m) == b_lo;
+        if (b_hi == b_lo) {  // the warp's rows in one sample: one gate row (warp-uniform)
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const float g0 = __shfl_sync(0xffffffffu, pg0, j), g1 = __shfl_sync(0xffffffffu, pg1, j);
-          v[j] *= lo ? g0 : g1;
+          for (int j = 0; j < 32; ++j) v[j] *= __shfl_sync(0xffffffffu, pg0, j);
+        } else {
+          const bool lo = m >= M || epi_batch(e, m) == b_lo;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float g0 = __shfl_sync(0xffffffffu, pg0, j), g1 = __shfl_sync(0xffffffffu, pg1, j);
+            v[j] *= lo ? g0 : g1;
+          }
         }
       }
       if (pre) {
