@@ -167,7 +167,8 @@ def test_gemm_plain_and_bias(cuda, dtype, M, N, K):
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("M,N,K,rpb", [(384, 256, 192, 128),      # row-wise epilogue
                                        (1100, 520, 192, 500),     # ragged: a swapped tile of 8 columns
-                                       (4096, 1152, 1152, 256)])  # DiT-XL/2 out-projection: 4 x 32 + 16 swapped tiles
+                                       (4096, 1152, 1152, 256),   # DiT-XL/2 out-projection: 4 x 32 + 16 swapped tiles
+                                       (512, 2048, 8192, 256)])   # K = 8192: CTA-pair tiles, staged epilogue
 def test_gemm_fused_epilogues(cuda, dtype, M, N, K, rpb):
     a = randn((M, K), dtype, 4)
     w = randn((N, K), dtype, 5, 0.08)
