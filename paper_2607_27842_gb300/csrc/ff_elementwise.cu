@@ -406,12 +406,13 @@ cudaError_t launch_ln_ab(DType dt, const float* mod, long long mod_stride, int r
 // One warp per row, the row held in registers (NCH 16-byte vectors per
 // lane): one global read, exact two-pass mean / variance, one write.
 // ---------------------------------------------------------------------------
-// One warp per row (8 rows per block); the block first stages the shift /
+// One warp per row (8 rows per block, for row counts that fill about two
+// waves at most); the block first stages the shift /
 // scale vectors of its first row's sample in shared memory (coalesced, read
 // back by every warp of that sample instead of 4 x 16 B per lane per chunk
 // from global memory).
 template <class T, int NCH>
-__global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
+__global__ void __launch_bounds__(256) k_ln_mod1(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
                                                 const float* __restrict__ shift, const float* __restrict__ scale,
                                                 int mod_stride, int seg_split, int rpb0, int rpb1) {
   pdl_trigger();
@@ -483,25 +484,138 @@ __global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __re
   }
 }
 
+// Each warp takes rpw rows (8 warps, a block of 8 * rpw consecutive rows);
+// the block first stages the shift / scale vectors of its first row's
+// sample in shared memory (coalesced, read back by every warp of that sample
+// instead of 4 x 16 B per lane per chunk from global memory); a warp loads
+// its next row while it reduces and writes the current one.
+template <class T, int NCH>
+__global__ void __launch_bounds__(256) k_ln_mod(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
+                                                const float* __restrict__ shift, const float* __restrict__ scale,
+                                                int mod_stride, int seg_split, int rpb0, int rpb1, int rpw) {
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ float4 smod4[];                  // [2 * C / 4]: shift, then scale
+  float* smod = reinterpret_cast<float*>(smod4);
+  constexpr int V = VecN<T>::n;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long r0 = (long long)blockIdx.x * 8 * rpw;
+  const int b0 = (int)(r0 < seg_split ? r0 / rpb0 : (r0 - seg_split) / rpb1);
+  const int nv = C / V;
+  // rows r0 + warp * rpw + t, t < rpw; the first one's loads go out before
+  // the staging
+  const long long rw = r0 + (long long)warp * rpw;
+  uint4 cur[NCH];
+  auto load_row = [&](long long r, uint4 (&v)[NCH]) {
+    const T* xr = x + r * C;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+      const int k = lane + 32 * j;
+      if (k < nv) v[j] = *reinterpret_cast<const uint4*>(xr + k * V);
+    }
+  };
+  if (rw < rows) load_row(rw, cur);
+  {
+    const float4* sh4 = reinterpret_cast<const float4*>(shift + (size_t)b0 * mod_stride);
+    const float4* sc4 = reinterpret_cast<const float4*>(scale + (size_t)b0 * mod_stride);
+    for (int i = threadIdx.x; i < C / 4; i += blockDim.x) {
+      smod4[i] = sh4[i];
+      smod4[C / 4 + i] = sc4[i];
+    }
+  }
+  __syncthreads();
+  for (int t = 0; t < rpw; ++t) {
+    const long long r = rw + t;
+    if (r >= rows) break;
+    uint4 nxt[NCH];
+    const bool more = t + 1 < rpw && r + 1 < rows;
+    if (more) load_row(r + 1, nxt);
+    float s = 0.f;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+      if (lane + 32 * j < nv) {
+        float a[V];
+        unpack16(cur[j], a);
+#pragma unroll
+        for (int q = 0; q < V; ++q) s += a[q];
+      }
+    }
+    s = warp_sum(s);
+    const float mean = s / C;
+    float ss = 0.f;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+      if (lane + 32 * j < nv) {
+        float a[V];
+        unpack16(cur[j], a);
+#pragma unroll
+        for (int q = 0; q < V; ++q) { const float d = a[q] - mean; ss += d * d; }
+      }
+    }
+    ss = warp_sum(ss);
+    const float rstd = rsqrtf(ss / C + 1e-6f);
+    const int b = (int)(r < seg_split ? r / rpb0 : (r - seg_split) / rpb1);
+    // the block's sample from shared memory, another sample (a block
+    // straddling a sample boundary) from global memory
+    const float* sh = b == b0 ? smod : shift + (size_t)b * mod_stride;
+    const float* sc = b == b0 ? smod + C : scale + (size_t)b * mod_stride;
+    T* orow = out + r * C;
+#pragma unroll
+    for (int j = 0; j < NCH; ++j) {
+      const int k = lane + 32 * j;
+      if (k < nv) {
+        float a[V], o[V];
+        unpack16(cur[j], a);
+#pragma unroll
+        for (int q = 0; q < V; q += 4) {
+          const float4 s4 = *reinterpret_cast<const float4*>(sh + k * V + q);
+          const float4 c4 = *reinterpret_cast<const float4*>(sc + k * V + q);
+          o[q] = (a[q] - mean) * rstd * (1.0f + c4.x) + s4.x;
+          o[q + 1] = (a[q + 1] - mean) * rstd * (1.0f + c4.y) + s4.y;
+          o[q + 2] = (a[q + 2] - mean) * rstd * (1.0f + c4.z) + s4.z;
+          o[q + 3] = (a[q + 3] - mean) * rstd * (1.0f + c4.w) + s4.w;
+        }
+        st16(orow + k * V, o);
+      }
+    }
+    if (more) {
+#pragma unroll
+      for (int j = 0; j < NCH; ++j) cur[j] = nxt[j];
+    }
+  }
+}
+
 template <class T>
 static cudaError_t ln_mod_t(const void* x, void* out, long long rows, int C, const float* shift, const float* scale,
                             int mod_stride, int seg_split, int rpb0, int rpb1, cudaStream_t s) {
   constexpr int V = VecN<T>::n;
   const int nch = (C / V + 31) / 32;
-  const unsigned grid = (unsigned)((rows + 7) / 8);
+  // rows per warp: one while a row per warp makes at most about two waves
+  // of blocks (every row's loads in flight at once), else enough that the
+  // blocks fill about two per SM (measured: 4096 x 1152 rows 6.6 us with one
+  // row per warp, 8.5 us with two; 14310 x 2048 rows 32.5 us with one, 24.5
+  // us with six)
+  const long long per_wave = 8LL * 2 * num_sms();
+  int rpw = rows <= 2 * per_wave ? 1 : (int)((rows + per_wave - 1) / per_wave);
+  rpw = rpw < 1 ? 1 : rpw > 8 ? 8 : rpw;
+  const unsigned grid = (unsigned)((rows + 8LL * rpw - 1) / (8LL * rpw));
   const size_t smem = (size_t)2 * C * sizeof(float);  // shift + scale of one sample
   if (C % 4 != 0 || smem > 48 * 1024) return cudaErrorInvalidValue;
   const T* xp = (const T*)x;
   T* op = (T*)out;
 #define FF_LN_CASE(n) \
-  case n: launch_pdl(k_ln_mod<T, n>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break;
-  switch (nch) {
+  case n:                                                                                                              \
+    if (rpw == 1)                                                                                                      \
+      launch_pdl(k_ln_mod1<T, n>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); \
+    else                                                                                                               \
+      launch_pdl(k_ln_mod<T, n>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1,  \
+                 rpw);                                                                                                 \
+    break;
+  const int nchr = nch <= 6 ? nch : nch <= 8 ? 8 : nch <= 12 ? 12 : nch <= 16 ? 16 : 0;
+  switch (nchr) {
     FF_LN_CASE(1) FF_LN_CASE(2) FF_LN_CASE(3) FF_LN_CASE(4) FF_LN_CASE(5) FF_LN_CASE(6)
     FF_LN_CASE(8) FF_LN_CASE(12) FF_LN_CASE(16)
     default:
-      if (nch <= 8) { launch_pdl(k_ln_mod<T, 8>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
-      if (nch <= 12) { launch_pdl(k_ln_mod<T, 12>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
-      if (nch <= 16) { launch_pdl(k_ln_mod<T, 16>, grid, 256, smem, s, xp, op, rows, C, shift, scale, mod_stride, seg_split, rpb0, rpb1); break; }
       return cudaErrorInvalidValue;
   }
 #undef FF_LN_CASE
