@@ -657,11 +657,18 @@ template <int BN> struct Cfg2 {
 
 // The epilogue is epi_tile's (staged TMA-store blocks where tm.staged), each
 // CTA on its own 128 rows of the pair's 256-row tile.
-template <int BN, int LN>
+// GROUPED: a second problem of the same N and K (its own A, W, rows,
+// epilogue and store maps: the text stream of a two-stream block beside the
+// image stream), its tiles first in the tile list, so its few tiles fill the
+// first problem's last wave instead of running alone on a handful of SMs.
+template <int BN, int LN, bool GROUPED>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     k_gemm_tc2(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                const __grid_constant__ CUtensorMap tmO, const __grid_constant__ CUtensorMap tmH, int M, int N, int K,
-               const __grid_constant__ TileMap tm, const __grid_constant__ EpiArgs e) {
+               const __grid_constant__ TileMap tm, const __grid_constant__ EpiArgs e,
+               const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+               const __grid_constant__ CUtensorMap tmO1, const __grid_constant__ CUtensorMap tmH1, int M1,
+               const __grid_constant__ TileMap tm1, const __grid_constant__ EpiArgs e1) {
   using C = Cfg2<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -680,7 +687,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   const bool leader = rank == 0;
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   const int num_m = (M + 2 * BM - 1) / (2 * BM), num_n = (N + BN - 1) / BN;
-  const int num_tiles = num_m * num_n;
+  const int num_m1 = GROUPED ? (M1 + 2 * BM - 1) / (2 * BM) : 0;
+  const int n1 = num_m1 * num_n;              // group 1's tiles come first
+  const int num_tiles = n1 + num_m * num_n;
+  // (group, row block, column block) of tile `tile`
+  auto tile_of = [&](int tile, bool& g1, int& mb, int& nb) {
+    g1 = GROUPED && tile < n1;
+    const int u = g1 ? tile : tile - n1;
+    const int nm = g1 ? num_m1 : num_m;
+    mb = u % nm;
+    nb = u / nm;
+  };
   const int num_kb = (K + BK - 1) / BK;
 
   if (threadIdx.x == 0) {
@@ -696,6 +713,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB) : "memory");
+    if (GROUPED && n1) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmA1) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&tmB1) : "memory");
+    }
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(tmem_slot)),
@@ -718,15 +739,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int tile = pair; tile < num_tiles && ok; tile += npairs) {
-        const int mb = tile % num_m, nb = tile / num_m;
+        bool g1;
+        int mb, nb;
+        tile_of(tile, g1, mb, nb);
         for (int kb = 0; kb < num_kb; ++kb, ++it) {
           const int s = it % C::STAGES;
           const uint32_t ph = (it / C::STAGES) & 1;
           if (!mbar_wait_p(&empty[s], ph ^ 1, abort_flag)) { ok = false; break; }
           if (leader) mbar_expect_tx(&full[s], 2 * C::STAGE_BYTES);
           const uint32_t fb = map_to(&full[s], 0);
-          tma_load_pair(&tmA, fb, sA + s * C::A_BYTES, kb * BK, mb * 2 * BM + (int)rank * BM);
-          tma_load_pair(&tmB, fb, sB + s * C::B_BYTES, kb * BK, nb * BN + (int)rank * C::HB);
+          // (each call names its kernel parameter: a tensor map stays in
+          // parameter space)
+          if (g1) {
+            tma_load_pair(&tmA1, fb, sA + s * C::A_BYTES, kb * BK, mb * 2 * BM + (int)rank * BM);
+            tma_load_pair(&tmB1, fb, sB + s * C::B_BYTES, kb * BK, nb * BN + (int)rank * C::HB);
+          } else {
+            tma_load_pair(&tmA, fb, sA + s * C::A_BYTES, kb * BK, mb * 2 * BM + (int)rank * BM);
+            tma_load_pair(&tmB, fb, sB + s * C::B_BYTES, kb * BK, nb * BN + (int)rank * C::HB);
+          }
         }
       }
       if (leader) {  // the even CTA's full barriers track both CTAs' copies
@@ -774,12 +804,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     int tc = 0;
     uint32_t epi_cnt = 0;
     for (int tile = pair; tile < num_tiles; tile += npairs, ++tc) {
-      const int mb = tile % num_m, nb = tile / num_m;
+      bool g1;
+      int mb, nb;
+      tile_of(tile, g1, mb, nb);
       const int acc = tc & 1;
       const uint32_t aph = (tc >> 1) & 1;
       const TileAt t = {false, mb * 2 * BM + (int)rank * BM, nb * BN};
-      if (!epi_tile<BN, C::XPOSE_BYTES, true, LN>(W, e, tm, M, N, t, acc, aph, epi_cnt, &tmO, &tmH, &tmO, &tmO))
-        break;
+      bool ok;
+      if (g1)
+        ok = epi_tile<BN, C::XPOSE_BYTES, true, LN>(W, e1, tm1, M1, N, t, acc, aph, epi_cnt, &tmO1, &tmH1, &tmO1,
+                                                     &tmO1);
+      else
+        ok = epi_tile<BN, C::XPOSE_BYTES, true, LN>(W, e, tm, M, N, t, acc, aph, epi_cnt, &tmO, &tmH, &tmO, &tmO);
+      if (!ok) break;
       tc_fence_before();
       mbar_arrive_cluster(map_to(&tempty[acc], 0));
     }
@@ -803,9 +840,9 @@ template <int BN, bool G>
 auto gemm_fn(int ln) -> decltype(&k_gemm_tc<BN, G, 0>) {
   return ln == 1 ? k_gemm_tc<BN, G, 1> : ln == 2 ? k_gemm_tc<BN, G, 2> : k_gemm_tc<BN, G, 0>;
 }
-template <int BN>
-auto gemm2_fn(int ln) -> decltype(&k_gemm_tc2<BN, 0>) {
-  return ln == 1 ? k_gemm_tc2<BN, 1> : ln == 2 ? k_gemm_tc2<BN, 2> : k_gemm_tc2<BN, 0>;
+template <int BN, bool G = false>
+auto gemm2_fn(int ln) -> decltype(&k_gemm_tc2<BN, 0, G>) {
+  return ln == 1 ? k_gemm_tc2<BN, 1, G> : ln == 2 ? k_gemm_tc2<BN, 2, G> : k_gemm_tc2<BN, 0, G>;
 }
 int ln_side(const EpiArgs& e) { return e.ln_in ? 1 : e.ln_out ? 2 : 0; }
 // a fused LayerNorm side: one side per launch, bf16 output of whole
@@ -846,6 +883,8 @@ bool init_driver() {
     for (int ln = 0; ln < 3; ++ln) {
       cudaFuncSetAttribute(gemm2_fn<128>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<128>::SMEM);
       cudaFuncSetAttribute(gemm2_fn<256>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<256>::SMEM);
+      cudaFuncSetAttribute(gemm2_fn<128, true>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<128>::SMEM);
+      cudaFuncSetAttribute(gemm2_fn<256, true>(ln), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg2<256>::SMEM);
     }
   });
   return g_encode != nullptr;
@@ -928,10 +967,13 @@ cudaError_t gemm_tc(int M, int N, int K, const void* A, int lda, const void* W, 
     TileMap tm2 = {};
     CUtensorMap mo = ma, mh = ma;
     tm2.staged = staged_maps(e, M, N, &mo, &mh) ? 1 : 0;
+    const TileMap none = {};
     if (bn == 256)
-      launch_pdl(gemm2_fn<256>(ln_side(e)), grid, THREADS, Cfg2<256>::SMEM, s, ma, mb, mo, mh, M, N, K, tm2, e);
+      launch_pdl(gemm2_fn<256>(ln_side(e)), grid, THREADS, Cfg2<256>::SMEM, s, ma, mb, mo, mh, M, N, K, tm2, e, ma, mb,
+                 mo, mh, 0, none, e);
     else
-      launch_pdl(gemm2_fn<128>(ln_side(e)), grid, THREADS, Cfg2<128>::SMEM, s, ma, mb, mo, mh, M, N, K, tm2, e);
+      launch_pdl(gemm2_fn<128>(ln_side(e)), grid, THREADS, Cfg2<128>::SMEM, s, ma, mb, mo, mh, M, N, K, tm2, e, ma, mb,
+                 mo, mh, 0, none, e);
     return launched();
   }
   // Every tile (128 x 256 full rate, 128 x 128 at half rate, swapped 128 x
@@ -1017,9 +1059,36 @@ cudaError_t gemm_tc_grouped(int M0, const void* A0, const void* W0, const EpiArg
   if (!init_driver()) return cudaErrorNotSupported;
   if (!ln_ok(e0, N) || !ln_ok(e1, N) || (ln_side(e0) && ln_side(e1) && ln_side(e0) != ln_side(e1)))
     return cudaErrorInvalidValue;
-  // CTA-pair reductions and column counts that need swapped tiles run as
-  // two launches
-  if ((M0 >= 2 * BM && K >= 8192) || N % 256 != 0) {
+  // long reductions: both problems in one CTA-pair launch (256-row tiles
+  // of the image rows, then of the text rows)
+  if (M0 >= 2 * BM && K >= 8192) {
+    if (K % 8 != 0 || lda % 8 != 0 || ldw % 8 != 0 || N % 8 != 0) return cudaErrorInvalidValue;
+    if (((uintptr_t)A0 & 15) || ((uintptr_t)W0 & 15) || ((uintptr_t)A1 & 15) || ((uintptr_t)W1 & 15))
+      return cudaErrorInvalidValue;
+    const int pairs = g_sms / 2;
+    const long long rows_t = ((M0 + 2 * BM - 1) / (2 * BM)) + ((M1 + 2 * BM - 1) / (2 * BM));
+    const int bn = pick_bn((int)(rows_t * 2 * BM), N, 2 * BM, pairs);
+    CUtensorMap a0, b0, a1, b1;
+    if (!make_map(&a0, A0, M0, K, lda, BM) || !make_map(&b0, W0, N, K, ldw, bn / 2) ||
+        !make_map(&a1, A1, M1, K, lda, BM) || !make_map(&b1, W1, N, K, ldw, bn / 2))
+      return cudaErrorInvalidValue;
+    TileMap t0 = {}, t1 = {};
+    CUtensorMap o0 = a0, h0 = a0, o1 = a1, h1 = a1;
+    t0.staged = staged_maps(e0, M0, N, &o0, &h0) ? 1 : 0;
+    t1.staged = staged_maps(e1, M1, N, &o1, &h1) ? 1 : 0;
+    const long long tiles = rows_t * ((N + bn - 1) / bn);
+    const int grid = 2 * (int)(tiles < pairs ? tiles : pairs);
+    const int ln = std::max(ln_side(e0), ln_side(e1));
+    if (bn == 256)
+      launch_pdl(gemm2_fn<256, true>(ln), grid, THREADS, Cfg2<256>::SMEM, s, a0, b0, o0, h0, M0, N, K, t0, e0, a1, b1, o1,
+                 h1, M1, t1, e1);
+    else
+      launch_pdl(gemm2_fn<128, true>(ln), grid, THREADS, Cfg2<128>::SMEM, s, a0, b0, o0, h0, M0, N, K, t0, e0, a1, b1, o1,
+                 h1, M1, t1, e1);
+    return launched();
+  }
+  // column counts that need swapped tiles run as two launches
+  if (N % 256 != 0) {
     const cudaError_t r = gemm_tc(M1, N, K, A1, lda, W1, ldw, e1, s);
     return r != cudaSuccess ? r : gemm_tc(M0, N, K, A0, lda, W0, ldw, e0, s);
   }
