@@ -394,6 +394,10 @@ static inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 b
 // launchers (return the launch error; work is asynchronous on `s`)
 // ---------------------------------------------------------------------------
 struct Hist4 { const void* p[4]; };
+// The history entries of a run of consecutive drafted blocks (at most
+// SEG_MAX blocks, K_eff + 1 entries each, newest first).
+constexpr int SEG_MAX = 64;
+struct HistSeg { const void* p[SEG_MAX][4]; };
 
 // Process-wide count of kernels this library has launched.
 void count_launches(long long n);
@@ -404,6 +408,11 @@ inline cudaError_t launched() {
 }
 
 cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int nt, long long n, cudaStream_t s);
+// x <- x + sum_{b < nblk} sum_j w_j h.p[b][j]: the per-block drafts of nblk
+// consecutive blocks (Eq. 2 with the same weights for every block) chained
+// in one pass, in fp32, rounded once.
+cudaError_t launch_draft_seg(DType dt, void* x, const HistSeg& h, int nblk, const float* w, int nt, long long n,
+                             cudaStream_t s);
 cudaError_t launch_diff(DType dt, const void* a, const void* b, void* out, long long n, cudaStream_t s);
 size_t verify_workspace_bytes(long long n);
 // Queries how many paid-check clusters are resident at once (the launched

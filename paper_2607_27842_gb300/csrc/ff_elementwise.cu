@@ -101,6 +101,66 @@ cudaError_t launch_draft(DType dt, void* x, const Hist4& h, const float* w, int 
   return dt == F32 ? draft_t<float>(x, h, w, nt, n, s) : draft_t<bf16>(x, h, w, nt, n, s);
 }
 
+// A run of nblk drafted blocks in one pass: x <- x + sum_b sum_j w_j R_{b,j}.
+// Each block's draft adds its forecast increment to the incoming state, so
+// the run's blocks telescope; x is read and written once instead of once
+// per block, and the sum stays in fp32 until the end.
+template <class T, int NT>
+__global__ void __launch_bounds__(256) k_draft_seg(T* __restrict__ x, const __grid_constant__ HistSeg h, int nblk,
+                                                   float w0, float w1, float w2, float w3, long long n) {
+  pdl_trigger();
+  pdl_wait();
+  constexpr int V = VecN<T>::n;
+  const float w[4] = {w0, w1, w2, w3};
+  const long long nvec = n / V;
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < nvec; i += stride) {
+    float a[V];
+    ld16(x + i * V, a);
+    for (int b = 0; b < nblk; ++b) {
+#pragma unroll
+      for (int j = 0; j < NT; ++j) {
+        float r[V];
+        ld16(reinterpret_cast<const T*>(h.p[b][j]) + i * V, r);
+#pragma unroll
+        for (int q = 0; q < V; ++q) a[q] = __fmaf_rn(w[j], r[q], a[q]);
+      }
+    }
+    st16(x + i * V, a);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < n - nvec * V) {
+    const long long i = nvec * V + threadIdx.x;
+    float a = to_f(x[i]);
+    for (int b = 0; b < nblk; ++b) {
+#pragma unroll
+      for (int j = 0; j < NT; ++j) a = __fmaf_rn(w[j], to_f(reinterpret_cast<const T*>(h.p[b][j])[i]), a);
+    }
+    x[i] = from_f<T>(a);
+  }
+}
+
+template <class T>
+static cudaError_t draft_seg_t(void* x, const HistSeg& h, int nblk, const float* w, int nt, long long n,
+                               cudaStream_t s) {
+  const int grid = stream_grid(n / VecN<T>::n, 256);
+  T* xp = reinterpret_cast<T*>(x);
+  switch (nt) {
+    case 1: launch_pdl(k_draft_seg<T, 1>, grid, 256, 0, s, xp, h, nblk, w[0], w[1], w[2], w[3], n); break;
+    case 2: launch_pdl(k_draft_seg<T, 2>, grid, 256, 0, s, xp, h, nblk, w[0], w[1], w[2], w[3], n); break;
+    case 3: launch_pdl(k_draft_seg<T, 3>, grid, 256, 0, s, xp, h, nblk, w[0], w[1], w[2], w[3], n); break;
+    case 4: launch_pdl(k_draft_seg<T, 4>, grid, 256, 0, s, xp, h, nblk, w[0], w[1], w[2], w[3], n); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return launched();
+}
+
+cudaError_t launch_draft_seg(DType dt, void* x, const HistSeg& h, int nblk, const float* w, int nt, long long n,
+                             cudaStream_t s) {
+  if (n <= 0 || nblk <= 0) return cudaSuccess;
+  if (nblk > SEG_MAX) return cudaErrorInvalidValue;
+  return dt == F32 ? draft_seg_t<float>(x, h, nblk, w, nt, n, s) : draft_seg_t<bf16>(x, h, nblk, w, nt, n, s);
+}
+
 // out = a - b elementwise (fp32 arithmetic, rounded to the storage type).
 template <class T>
 __global__ void __launch_bounds__(256) k_diff(const T* __restrict__ a, const T* __restrict__ b, T* __restrict__ out,

@@ -850,6 +850,22 @@ featfix_status verify_shadow(featfix_ctx* ctx, int i, int nt, const float* wf) {
                           ctx->dsums + 4 * slot, ctx->vws, ctx->st, nullptr, verify_counter(ctx)));
       ctx->log_sites.push_back({i, l});
     } else {
+      // the run of drafted blocks up to the next site in one pass, as the
+      // FeatFix arm's site steps do (so both arms reach their first site
+      // with the same state)
+      int l2 = l + 1;
+      while (l2 <= last && l2 - l < SEG_MAX && ctx->kinds[(size_t)i * L + l2] == FEATFIX_PLAN_DRAFT) ++l2;
+      if (l2 - l > 1) {
+        HistSeg hs = {};
+        for (int b = l; b < l2; ++b) {
+          const Hist4 hp = hist_ptrs(ctx, b, nt);
+          for (int j = 0; j < 4; ++j) hs.p[b - l][j] = hp.p[j];
+        }
+        KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt * (l2 - l) + 2) * bytes);
+        FF_CK(launch_draft_seg(ctx->dt, ctx->shadow, hs, l2 - l, wf, nt, ctx->E, ctx->st));
+        l = l2 - 1;
+        continue;
+      }
       KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
       FF_CK(launch_draft(ctx->dt, ctx->shadow, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
     }
@@ -891,6 +907,8 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
   for (auto& cp : ctx->caps) has_capture |= cp.step == i;
   const bool telescope = !refresh && !vanilla && !has_capture && !site_push &&
                          !(ctx->flags & FEATFIX_FLAG_PER_BLOCK_DRAFT) && (!has_site || ctx->mode == FEATFIX_MODE_VERIFY);
+  // drafted blocks between the sites of a per-block step: one pass per run
+  const bool seg_ok = !site_push && !has_capture && !(ctx->flags & FEATFIX_FLAG_PER_BLOCK_DRAFT);
   void* x = ctx->x0buf;
   if (telescope) {
     if (has_site) FF_TRY(verify_shadow(ctx, i, nt, wf));
@@ -925,6 +943,22 @@ featfix_status step_body(featfix_ctx* ctx, float* latent, int i, const void* con
         advance();
       } else if (kind == FEATFIX_PLAN_DRAFT) {
         block_weights(l);
+        // a run of drafted blocks in one pass (same weights for every block;
+        // per block with site pushes, captures or FEATFIX_FLAG_PER_BLOCK_DRAFT)
+        int l2 = l + 1;
+        if (seg_ok)
+          while (l2 < L && l2 - l < SEG_MAX && ctx->kinds[(size_t)i * L + l2] == FEATFIX_PLAN_DRAFT) ++l2;
+        if (l2 - l > 1) {
+          HistSeg hs = {};
+          for (int b = l; b < l2; ++b) {
+            const Hist4 hp = hist_ptrs(ctx, b, nt);
+            for (int j = 0; j < 4; ++j) hs.p[b - l][j] = hp.p[j];
+          }
+          KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt * (l2 - l) + 2) * bytes);
+          FF_CK(launch_draft_seg(ctx->dt, x, hs, l2 - l, wf, nt, ctx->E, ctx->st));
+          l = l2 - 1;
+          continue;
+        }
         KTimer tm(ctx, FEATFIX_KCLASS_DRAFT, (double)(nt + 2) * bytes);
         FF_CK(launch_draft(ctx->dt, x, hist_ptrs(ctx, l, nt), wf, nt, ctx->E, ctx->st));
       } else {

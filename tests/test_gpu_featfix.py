@@ -80,9 +80,10 @@ def test_sample_matches_oracle(case, mode):
     lat2 = case.sample(seed=1)
     logs2, _ = ff.featfix_get_log(case.ctx)
     case.check_logs_teacher_forced(bufs, logs2, mode)
-    # captures take site steps block by block (the default for FeatFix)
-    if mode == "featfix":
-        assert torch.equal(lat, lat2) and logs2 == logs
+    # with captures a site step's drafted blocks are chained one by one
+    # instead of in one pass per run of blocks: the same value up to rounding
+    assert [(e["step"], e["layer"]) for e in logs2] == [(e["step"], e["layer"]) for e in logs]
+    assert rel_l2(lat2.cpu().numpy(), lat.cpu().numpy()) < (1e-5 if case.sh.dtype == "f32" else 1e-2)
     ff.featfix_debug_capture(case.ctx, -1, 0, None, None)
 
 
