@@ -56,6 +56,8 @@ def parse():
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--mode", default="featfix", choices=["featfix", "verify", "exact_only", "vanilla"])
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--stepwise", action="store_true",
+                   help="also time the same runs driven one featfix_step call per denoising step (no whole-run graph)")
     p.add_argument("--cpu-leg", type=int, default=0, help=argparse.SUPPRESS)   # internal: oracle timing process
     p.add_argument("--sweep", choices=["resolution"], default=None,
                    help="instead of the headline line: one line per FLUX resolution (512^2, 768^2, 1024^2) with "
@@ -523,6 +525,25 @@ def main():
     barrier()
     e2e_s = time.perf_counter() - t0
 
+    # ---- optional: the same runs driven one featfix_step call per denoising step ----
+    step_ms = None
+    if args.stepwise:
+        x = torch.empty(sh.latent_dims, dtype=torch.float32, device=dev)
+        for i in range(args.warmup):
+            x.normal_()
+            for t in range(wl.steps):
+                ff.featfix_step(ctx, x, t, cond)
+        barrier()
+        ev2, ev3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev2.record(stream)
+        for i in range(args.steps):
+            x.normal_()
+            for t in range(wl.steps):
+                ff.featfix_step(ctx, x, t, cond)
+        ev3.record(stream)
+        barrier()
+        step_ms = ev2.elapsed_time(ev3)
+
     ms_max, e2e_max = slowest_rank(dist, [ms, e2e_s], dev)
     value = job_rate(args.steps * wl.steps, world, ms_max / 1e3)
     e2e = job_rate(args.steps * wl.steps, world, e2e_max)
@@ -542,6 +563,10 @@ def main():
         "counters": counters,
         "clocks": clk,
     }
+    if step_ms is not None:
+        line["stepwise"] = {"value": job_rate(args.steps * wl.steps, 1, step_ms / 1e3), "unit": UNIT,
+                            "how": "one featfix_step call per denoising step from the host (no whole-run CUDA "
+                                   "graph), the same runs, CUDA events (latent re-initialised with normal_ per run)"}
     if want_cpu:
         one_core = finish_cpu_leg(leg1, wl)
         line["cpu_baseline"] = finish_cpu_leg(start_cpu_leg(wl, all_cores()), wl)
