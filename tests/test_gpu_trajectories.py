@@ -20,7 +20,8 @@ the full workloads'.  Checked per trajectory (Section 3.3, Eqs. 2-5): the
 final latent within 5e-2 relative L2 (bf16), the paid checks in the same
 order, the accounting bit-exact, and every logged discrepancy against Eq. 4
 evaluated by the oracle on the GPU's own captured tensors (2e-2).  The
-FeatFix arm runs again with every drafted step chained block by block.
+FeatFix arm runs again with every drafted step chained block by block, and
+with the adaLN LayerNorm fused across the dense layers.
 """
 
 import importlib.util
@@ -87,5 +88,9 @@ def test_trajectory_matches_stored_oracle(cuda, name, mode):
             lat3 = c.sample(seed=gm.SEED_LATENT)
             assert rel_l2(lat3.cpu().numpy(), x_ref) < tol_latent(c.sh)
             assert not torch.equal(lat3, lat)
+            # the adaLN LayerNorm fused across the dense layers (opt-in)
+            c.schedule(mode, flags=ff.FLAG_FUSED_LN)
+            lat4 = c.sample(seed=gm.SEED_LATENT)
+            assert rel_l2(lat4.cpu().numpy(), x_ref) < tol_latent(c.sh)
     finally:
         c.close()
