@@ -472,7 +472,7 @@ cudaError_t launch_ln_ab(DType dt, const float* mod, long long mod_stride, int r
 // back by every warp of that sample instead of 4 x 16 B per lane per chunk
 // from global memory).
 template <class T, int NCH>
-__global__ void __launch_bounds__(256) k_ln_mod1(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
+__global__ void __launch_bounds__(256, NCH <= 6 ? 4 : 1) k_ln_mod1(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
                                                 const float* __restrict__ shift, const float* __restrict__ scale,
                                                 int mod_stride, int seg_split, int rpb0, int rpb1) {
   pdl_trigger();
