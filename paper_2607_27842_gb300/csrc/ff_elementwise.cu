@@ -233,7 +233,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 // elsewhere; mix may be the h_f buffer itself (each element is read, then
 // written, by the same thread).
 template <class T, int NT>
-__global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_THREADS)
+__global__ void __cluster_dims__(VERIFY_CLUSTER, 1, 1) __launch_bounds__(VERIFY_THREADS, 4)
     k_verify(T* __restrict__ u, Hist4 h, float w0, float w1, float w2, float w3, const T* hf,
              long long n, int write_draft, double* __restrict__ partials, T* mix,
              const unsigned char* __restrict__ rmask, const unsigned char* __restrict__ cmask, int C,
