@@ -470,7 +470,8 @@ cudaError_t launch_ln_ab(DType dt, const float* mod, long long mod_stride, int r
 // waves at most); the block first stages the shift /
 // scale vectors of its first row's sample in shared memory (coalesced, read
 // back by every warp of that sample instead of 4 x 16 B per lane per chunk
-// from global memory).
+// from global memory).  Rows of up to six vectors per lane are held to 64
+// registers, so four blocks share an SM (4096 rows of 1152: one wave).
 template <class T, int NCH>
 __global__ void __launch_bounds__(256, NCH <= 6 ? 4 : 1) k_ln_mod1(const T* __restrict__ x, T* __restrict__ out, long long rows, int C,
                                                 const float* __restrict__ shift, const float* __restrict__ scale,
