@@ -22,6 +22,11 @@ with CUDA events and divides its algorithmic work by the summed time;
 Multi-GPU: replicas only (independent samples per GPU, no collective on the
 data path); the barrier and max-over-ranks timing use torch.distributed.
 
+Beside the cached rate the line carries the all-exact (vanilla) rate on the
+same GPU (``vanilla``; ``--no-vanilla`` skips it) and the paper's own
+latencies for the backbone the workload is shaped like (``paper``: context,
+hardware not stated).
+
 ``--impl reference`` times the CPU oracle on the host cores instead (a bounded
 sample of the same workload, extrapolated by the plan's counts).
 """
@@ -56,6 +61,8 @@ def parse():
     p.add_argument("--workload", default=WORKLOAD)
     p.add_argument("--mode", default="featfix", choices=["featfix", "verify", "exact_only", "vanilla"])
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-vanilla", action="store_true",
+                   help="skip the all-exact (vanilla) runs measured beside the cached rate")
     p.add_argument("--stepwise", action="store_true",
                    help="also time the same runs driven one featfix_step call per denoising step (no whole-run graph)")
     p.add_argument("--cpu-leg", type=int, default=0, help=argparse.SUPPRESS)   # internal: oracle timing process
@@ -286,6 +293,42 @@ def finish_cpu_leg(proc, wl, timeout_s=600):
 
 def all_cores():
     return os.cpu_count() or 1
+
+
+def host_cpu():
+    """The host the oracle legs run on: logical CPUs and the CPU model."""
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    import platform
+    return {"nproc": all_cores(), "cpu": model or platform.processor() or None, "machine": platform.machine()}
+
+
+# The paper's own latencies for the backbone each workload is shaped like
+# (real checkpoints, prompts and resolutions; hardware, precision and batch
+# not stated): context beside the measured rates, not a target.
+PAPER = {
+    "flux": {"backbone": "FLUX.1-dev, DrawBench200", "source": "Table 1", "vanilla_s": 23.93,
+             "featfix_s": [7.57, 4.76, 3.57], "speedup": [3.16, 5.03, 6.70]},
+    "qwen": {"backbone": "Qwen-Image, DrawBench200", "source": "Table 4", "vanilla_s": 22.59,
+             "featfix_s": [15.08, 10.40], "speedup": [1.50, 2.17]},
+    "hunyuan": {"backbone": "HunyuanVideo-1.5, 65 frames", "source": "Table 3", "vanilla_s": 772.60,
+                "featfix_s": [483.50, 415.10, 338.40], "speedup": [1.60, 1.86, 2.28]},
+    "dit_xl2": {"backbone": "DiT-XL/2, ImageNet-256", "source": "Table 5", "vanilla_s": 1.52,
+                "featfix_s": [0.45], "speedup": [3.38]},
+}
+
+
+def paper_context(wl):
+    base = wl.shape.name.split("_")[0] if wl.shape.name not in PAPER else wl.shape.name
+    rec = PAPER.get(base)
+    return dict(rec, hardware="not stated") if rec else None
 
 
 def run_reference(args, wl, rank):
@@ -544,6 +587,27 @@ def main():
         barrier()
         step_ms = ev2.elapsed_time(ev3)
 
+    # ---- the all-exact (vanilla) rate on the same GPU, weights and inputs ----
+    vanilla = None
+    if args.mode != "vanilla" and not args.no_vanilla and world == 1:
+        try:
+            nv = 2
+            ff.featfix_set_schedule(ctx, wl.steps, wl.refresh, wl.K, wl.sites, "vanilla")
+            ff.featfix_sample(ctx, 2000, wl.steps, cond, lat)   # untimed: builds the vanilla graph
+            barrier()
+            ev4, ev5 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            ev4.record(stream)
+            for i in range(nv):
+                ff.featfix_sample(ctx, 2001 + i, wl.steps, cond, lat)
+            ev5.record(stream)
+            barrier()
+            v_rate = job_rate(nv * wl.steps, 1, ev4.elapsed_time(ev5) / 1e3)
+            vanilla = {"value": v_rate, "unit": UNIT, "runs": nv, "cached_over_vanilla": None,
+                       "how": "the same context rescheduled with every block exact at every step, one untimed "
+                              "run, then %d runs timed with CUDA events" % nv}
+        except Exception as e:  # reported, never fatal for the cached number
+            vanilla = {"value": None, "unit": UNIT, "error": str(e)}
+
     ms_max, e2e_max = slowest_rank(dist, [ms, e2e_s], dev)
     value = job_rate(args.steps * wl.steps, world, ms_max / 1e3)
     e2e = job_rate(args.steps * wl.steps, world, e2e_max)
@@ -563,6 +627,13 @@ def main():
         "counters": counters,
         "clocks": clk,
     }
+    if vanilla is not None:
+        if vanilla.get("value"):
+            vanilla["cached_over_vanilla"] = value / vanilla["value"]
+        line["vanilla"] = vanilla
+    paper = paper_context(wl)
+    if paper is not None:
+        line["paper"] = paper
     if step_ms is not None:
         line["stepwise"] = {"value": job_rate(args.steps * wl.steps, 1, step_ms / 1e3), "unit": UNIT,
                             "how": "one featfix_step call per denoising step from the host (no whole-run CUDA "
@@ -571,6 +642,7 @@ def main():
         one_core = finish_cpu_leg(leg1, wl)
         line["cpu_baseline"] = finish_cpu_leg(start_cpu_leg(wl, all_cores()), wl)
         line["cpu_baseline_1core"] = one_core
+        line["cpu_baseline"]["host"] = host_cpu()
     ff.featfix_destroy(ctx)
     if rank == 0:
         print(json.dumps(line), flush=True)
