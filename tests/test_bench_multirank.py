@@ -51,3 +51,18 @@ def test_max_over_ranks_and_whole_job_rate():
 def test_single_rank_is_identity():
     assert bench.slowest_rank(None, [4.0, 5.0], "cpu") == [4.0, 5.0]
     assert bench.job_rate(50, 1, 0.1) == pytest.approx(500.0)
+
+
+def test_paper_context_is_consistent():
+    """The quoted speedups are the quoted latencies' ratios (Tables 1, 3, 4
+    and 5), and every bf16 workload maps to its backbone's record."""
+    from paper_2607_27842_gb300 import synthetic as syn
+    for rec in bench.PAPER.values():
+        assert len(rec["featfix_s"]) == len(rec["speedup"])
+        for t, sp in zip(rec["featfix_s"], rec["speedup"]):
+            assert abs(rec["vanilla_s"] / t - sp) < 0.006 * sp
+    assert bench.paper_context(syn.workload("tiny")) is None
+    for name, src in [("dit_xl2", "Table 5"), ("flux", "Table 1"), ("flux_512", "Table 1"), ("qwen", "Table 4"),
+                      ("qwen_512", "Table 4"), ("hunyuan", "Table 3"), ("hunyuan_3f", "Table 3")]:
+        rec = bench.paper_context(syn.workload(name))
+        assert rec["source"] == src and rec["hardware"] == "not stated"
