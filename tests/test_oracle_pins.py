@@ -107,6 +107,34 @@ def test_rope_axes_and_frequencies():
     np.testing.assert_allclose(ang[0], [2.0, 2.0 * 10000 ** -0.5, 5.0, 5.0 * 10000 ** -0.5])
 
 
+def test_patch_grid_and_image_positions_row_major():
+    """The image tokens' grid positions: last axis fastest (2-D: row, column;
+    3-D: frame, row, column), written out by hand for small grids, and the
+    grids of the video and image workloads."""
+    np.testing.assert_array_equal(model.image_positions((2, 3)),
+                                  [[0, 0], [0, 1], [0, 2], [1, 0], [1, 1], [1, 2]])
+    np.testing.assert_array_equal(model.image_positions((2, 1, 2)),
+                                  [[0, 0, 0], [0, 0, 1], [1, 0, 0], [1, 0, 1]])
+    assert model.patch_grid(synthetic.SHAPES["hunyuan"]) == ((9, 30, 53), 4)
+    assert model.patch_grid(synthetic.SHAPES["flux"]) == ((64, 64), 4)
+    assert model.patch_grid(synthetic.SHAPES["dit_xl2"]) == ((16, 16), 4)
+
+
+def test_rope_table_of_a_video_token():
+    """3-D rotary angles of one image token (frame 2, row 1, column 4 of a
+    3 x 2 x 5 grid, token 2*10 + 1*5 + 4 = 29): the 16 / 56 / 56 axis split of
+    a 128-wide head, pair j of an axis of width w turning by
+    position * 10000^(-2j / w)."""
+    sh = synthetic.reduced(synthetic.SHAPES["hunyuan"], lat_f=3, lat_h=4, lat_w=10)
+    ang = model.rope_table(sh)
+    assert ang.shape == (30, 64)
+    a = ang[29]
+    for off, width, pos in ((0, 16, 2.0), (8, 56, 1.0), (36, 56, 4.0)):
+        for j in range(width // 2):
+            assert a[off + j] == pytest.approx(pos * 10000.0 ** (-2.0 * j / width), rel=1e-12)
+    assert model.rope_table(synthetic.SHAPES["dit_xl2"]) is None
+
+
 # ----------------------------------------------------------------------------
 # embeddings and layout
 # ----------------------------------------------------------------------------
