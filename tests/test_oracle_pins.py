@@ -463,6 +463,20 @@ def test_ddim_recovers_data_from_true_noise():
     np.testing.assert_allclose(x, x0, rtol=1e-9, atol=1e-9)
 
 
+def test_model_time_fed_to_the_embedding():
+    """Euler: t_i = 1000 sigma_i with sigma_i = 1 - i / N (1000 at the first
+    step, 1000 / N at the last); DDIM: the visited timestep 1000 - 20 (i + 1)
+    at N = 50.  Straight-path exactness and DDIM recovery hold for any time
+    map, so the map itself is pinned here."""
+    assert sampler.model_time("euler", 50, 0) == 1000.0
+    assert sampler.model_time("euler", 50, 49) == pytest.approx(20.0)
+    assert sampler.model_time("euler", 10, 5) == pytest.approx(500.0)
+    for i in (0, 7, 49):
+        assert sampler.model_time("ddim", 50, i) == 1000 - 20 * (i + 1)
+    sig = sampler.euler_sigmas(4)
+    np.testing.assert_allclose(sig, [1.0, 0.75, 0.5, 0.25, 0.0])
+
+
 def test_guidance_limits():
     out = rnd(4, 3)
     np.testing.assert_allclose(sampler.guide(out, 2, True, 1.0), out[:2])
