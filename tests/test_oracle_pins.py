@@ -425,6 +425,24 @@ def test_schedule_rules(bad):
         schedule.build_plan(args["steps"], args["L"], args["refresh"], args["K"], args["sites"], "featfix")
 
 
+def test_history_entries_by_hand():
+    """The refresh steps a draft reads (newest first, at most K + 1 = 2) on
+    the tiny schedule (refreshes 0, 3, 6, 9; sites (4, 2), (7, 1)), written
+    out from Section 3.3's rules: refreshes push every block; a site pushes
+    its own block only with the site-history reading (reading 5)."""
+    steps, L, ref, K, sites = 10, 4, (0, 3, 6, 9), 1, ((4, 2), (7, 1))
+    h = schedule.block_history_steps(steps, L, ref, K, sites, "featfix")
+    assert h[0] == [None] * 4 and h[3] == [None] * 4
+    assert h[1] == [[0]] * 4 and h[2] == [[0]] * 4
+    assert h[4] == [[3, 0]] * 4                  # the site (4, 2) drafts from the same entries
+    assert h[5][2] == [3, 0] and h[8] == [[6, 3]] * 4
+    hs = schedule.block_history_steps(steps, L, ref, K, sites, "featfix", site_updates_history=True)
+    assert hs[4][2] == [3, 0] and hs[5][2] == [4, 3] and hs[5][1] == [3, 0]
+    assert hs[7][1] == [6, 3] and hs[8][1] == [7, 6]
+    assert hs[7][2] == [6, 4] and hs[8][2] == [6, 4]  # the site's entry 4 outlives refresh 3
+    assert schedule.block_history_steps(steps, L, ref, K, sites, "vanilla")[5] == [None] * 4
+
+
 def test_vanilla_plan_is_all_exact():
     kind, _ = schedule.build_plan(6, 3, (0, 3), 1, ((1, 1),), "vanilla")
     assert all(k == schedule.EXACT for row in kind for k in row)
