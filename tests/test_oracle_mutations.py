@@ -1,0 +1,121 @@
+"""The oracle pins catch plausible mistakes: each case plants one mistake in a
+temporary copy of ``oracle/`` (a dropped term, a wrong sign, index or
+operand order, a swapped reading), runs the pins of
+``tests/test_oracle_pins.py`` against the copy in a fresh interpreter, and
+requires at least one of them to fail.  The unmodified copy passes.  The
+mistakes live only in the temporary copy; nothing here touches a GPU."""
+
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+# (file, text, replacement, pins to run (-k), what the mistake is)
+MUTATIONS = [
+    ("model.py", "return (x - mu) / np.sqrt(var + LN_EPS)", "return x / np.sqrt(var + LN_EPS)",
+     "layer_norm", "LayerNorm without the mean"),
+    ("model.py", "return x * (1.0 + scale[:, None, :]) + shift[:, None, :]",
+     "return x * (1.0 + shift[:, None, :]) + scale[:, None, :]",
+     "block", "shift and scale swapped"),
+    ("model.py", "(x + 0.044715 * x ** 3)", "(x + 0.044715 * x ** 2)",
+     "gelu", "GELU's cubic term squared"),
+    ("model.py", "out[..., 1::2] = x1 * s + x2 * c", "out[..., 1::2] = -x1 * s + x2 * c",
+     "rope", "rotary embedding with a sign error"),
+    ("model.py", "scale = 1.0 / np.sqrt(d)", "scale = 1.0 / d",
+     "attention", "attention scaled by 1/d"),
+    ("model.py", "e = linear(silu(linear(s, W[\"t_fc1.w\"], W[\"t_fc1.b\"])), W[\"t_fc2.w\"], W[\"t_fc2.b\"])",
+     "e = linear(linear(s, W[\"t_fc1.w\"], W[\"t_fc1.b\"]), W[\"t_fc2.w\"], W[\"t_fc2.b\"])",
+     "cond_vector", "SiLU dropped from the time MLP"),
+    ("model.py", "y = linear(modulate(layer_norm(tok), shift, scale), W[\"final.lin.w\"], W[\"final.lin.b\"])",
+     "y = linear(modulate(tok, shift, scale), W[\"final.lin.w\"], W[\"final.lin.b\"])",
+     "final_layer", "LayerNorm dropped from the final layer"),
+    ("model.py", "return np.concatenate([np.asarray(txt, dtype=np.float64), img], axis=1)",
+     "return np.concatenate([img, np.asarray(txt, dtype=np.float64)], axis=1)",
+     "embed_tokens", "text tokens after the image tokens"),
+    ("model.py", "u1 = u + g1[:, None, :] * linear(o, W[pre + \"proj.w\"], W[pre + \"proj.b\"])",
+     "u1 = u + g2[:, None, :] * linear(o, W[pre + \"proj.w\"], W[pre + \"proj.b\"])",
+     "dit_block", "the MLP gate on the attention branch"),
+    ("model.py", "idx = np.indices(grid).reshape(len(grid), -1).T",
+     "idx = np.indices(grid[::-1]).reshape(len(grid), -1).T[:, ::-1]",
+     "image_positions or rope_table", "image positions in column-major order"),
+    ("draft.py", "out = out + (t - s[0]) ** k / math.factorial(k) * Dk", "out = out + (t - s[0]) ** k * Dk",
+     "draft or order", "factorial dropped from the Taylor series"),
+    ("sampler.py", "return x + (sig[i + 1] - sig[i]) * v", "return x + (sig[i] - sig[i + 1]) * v",
+     "euler", "Euler step with the wrong sign"),
+    ("sampler.py", "return ou + scale * (oc - ou)", "return oc + scale * (oc - ou)",
+     "guidance", "guidance around the conditional output"),
+    ("sampler.py", "return euler_update(x, g[:, :shape.in_ch], steps, i)",
+     "return euler_update(x, g[:, -shape.in_ch:], steps, i)",
+     "step_update", "the velocity read from the wrong channels"),
+    ("sampler.py", "return 1000.0 * euler_sigmas(steps)[i]", "return 1000.0 * euler_sigmas(steps)[i + 1]",
+     "model_time", "the model time one step late"),
+    ("schedule.py", "k_eff.append(min(K, r - 1))", "k_eff.append(min(K, r))",
+     "plan or schedule", "draft order not limited by the refreshes seen"),
+    ("featfix.py", "                        h = hd\n", "                        h = hf\n",
+     "verify", "the Verify arm forwarding the exact output"),
+    ("featfix.py", "return float(np.abs(hd - hf).sum() / (np.abs(hf).sum() + EPS))",
+     "return float(np.abs(hd - hf).sum() / (np.abs(hd).sum() + EPS))",
+     "discrepancy", "Eq. 4 normalised by the draft"),
+]
+
+
+def _copy(tmp):
+    """The pins and what they import: tests (with the golden texts), the
+    oracle, and the input generator of the package."""
+    shutil.copytree(os.path.join(ROOT, "oracle"), os.path.join(tmp, "oracle"),
+                    ignore=shutil.ignore_patterns("__pycache__"))
+    os.makedirs(os.path.join(tmp, "tests", "golden"))
+    for f in ("__init__.py", "conftest.py", "test_oracle_pins.py"):
+        shutil.copy(os.path.join(ROOT, "tests", f), os.path.join(tmp, "tests", f))
+    for f in os.listdir(os.path.join(ROOT, "tests", "golden")):
+        if f.endswith(".txt"):
+            shutil.copy(os.path.join(ROOT, "tests", "golden", f), os.path.join(tmp, "tests", "golden", f))
+    pkg = os.path.join(tmp, "paper_2607_27842_gb300")
+    os.makedirs(pkg)
+    # the pins need the seeded generators and the weight names of the binding
+    # module (its library is never loaded)
+    with open(os.path.join(pkg, "__init__.py"), "w") as f:
+        f.write("")
+    for f in ("synthetic.py", "featfix.py"):
+        shutil.copy(os.path.join(ROOT, "paper_2607_27842_gb300", f), os.path.join(pkg, f))
+
+
+def _run_pins(tmp, select):
+    env = dict(os.environ, PYTHONDONTWRITEBYTECODE="1", OMP_NUM_THREADS="2", OPENBLAS_NUM_THREADS="2")
+    cmd = [sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider", "-m", "not gpu",
+           os.path.join("tests", "test_oracle_pins.py")]
+    if select:
+        cmd += ["-k", select]
+    return subprocess.run(cmd, cwd=tmp, env=env, capture_output=True, text=True, timeout=600)
+
+
+@pytest.fixture(scope="module")
+def pristine(tmp_path_factory):
+    tmp = str(tmp_path_factory.mktemp("oracle_copy"))
+    _copy(tmp)
+    return tmp
+
+
+def test_unmodified_copy_passes(pristine):
+    r = _run_pins(pristine, None)
+    assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-3000:]
+
+
+@pytest.mark.parametrize("fname,old,new,select,what", MUTATIONS, ids=[m[4] for m in MUTATIONS])
+def test_planted_mistake_fails_a_pin(tmp_path, fname, old, new, select, what):
+    tmp = str(tmp_path)
+    _copy(tmp)
+    path = os.path.join(tmp, "oracle", fname)
+    with open(path) as f:
+        src = f.read()
+    assert src.count(old) == 1, "the text to change must occur once in oracle/%s" % fname
+    with open(path, "w") as f:
+        f.write(src.replace(old, new))
+    r = _run_pins(tmp, select)
+    out = r.stdout + r.stderr
+    assert "no tests ran" not in out, out[-2000:]
+    assert r.returncode == 1, "%s: no pin failed\n%s" % (what, out[-3000:])
