@@ -55,6 +55,22 @@ MUTATIONS = [
      "model_time", "the model time one step late"),
     ("schedule.py", "k_eff.append(min(K, r - 1))", "k_eff.append(min(K, r))",
      "plan or schedule", "draft order not limited by the refreshes seen"),
+    ("model.py", "p /= p.sum(axis=-1, keepdims=True)", "p /= p.sum(axis=-2, keepdims=True)",
+     "attention", "softmax normalised over the queries"),
+    ("model.py", "return np.concatenate([np.cos(args), np.sin(args)])",
+     "return np.concatenate([np.sin(args), np.cos(args)])",
+     "sinusoid", "timestep features in [sin | cos] order"),
+    ("model.py", "rows, cols = np.meshgrid(np.arange(gh), np.arange(gw), indexing=\"ij\")",
+     "cols, rows = np.meshgrid(np.arange(gh), np.arange(gw), indexing=\"ij\")",
+     "sincos", "position rows and columns swapped"),
+    ("model.py", "qkv_t = linear(modulate(layer_norm(txt), mt[0], mt[1]), W[pre + \"txt_qkv.w\"], W[pre + \"txt_qkv.b\"])",
+     "qkv_t = linear(modulate(layer_norm(txt), mi[0], mi[1]), W[pre + \"txt_qkv.w\"], W[pre + \"txt_qkv.b\"])",
+     "dual_block", "the text stream modulated by the image stream's vectors"),
+    ("model.py", "out = linear(np.concatenate([o, gelu_tanh(mlp)], axis=-1), W[pre + \"lin2.w\"], W[pre + \"lin2.b\"])",
+     "out = linear(np.concatenate([gelu_tanh(mlp), o], axis=-1), W[pre + \"lin2.w\"], W[pre + \"lin2.b\"])",
+     "single_block", "the single block's [attention | MLP] order reversed"),
+    ("noise.py", "z = (z ^ (z >> np.uint64(27))) * M2", "z = (z ^ (z >> np.uint64(28))) * M2",
+     "splitmix", "a SplitMix64 shift off by one"),
     ("featfix.py", "                        h = hd\n", "                        h = hf\n",
      "verify", "the Verify arm forwarding the exact output"),
     ("featfix.py", "return float(np.abs(hd - hf).sum() / (np.abs(hf).sum() + EPS))",
