@@ -71,6 +71,15 @@ MUTATIONS = [
      "single_block", "the single block's [attention | MLP] order reversed"),
     ("noise.py", "z = (z ^ (z >> np.uint64(27))) * M2", "z = (z ^ (z >> np.uint64(28))) * M2",
      "splitmix", "a SplitMix64 shift off by one"),
+    ("schedule.py", "        if i in rs:\n            raise ScheduleError(\"site on a refresh step\")\n", "",
+     "schedule_rules", "a site on a refresh step accepted"),
+    ("draft.py", "table = [(table[j] - table[j + 1]) / (s[j] - s[j + m]) for j in range(n - m)]",
+     "table = [(table[j] - table[j + 1]) / (s[j] - s[j + 1]) for j in range(n - m)]",
+     "draft or order or taylor", "divided differences over the wrong node span"),
+    ("draft.py", "D[k] = D[k] + math.factorial(k) * coef[k] * dd[m]", "D[k] = D[k] + coef[k] * dd[m]",
+     "draft or order or taylor", "derivative estimates without k!"),
+    ("featfix.py", "hist[l].insert(0, (i, h - u))", "hist[l].insert(0, (i, h))",
+     "identity_blocks", "the block outputs forecast instead of their increments"),
     ("featfix.py", "                        h = hd\n", "                        h = hf\n",
      "verify", "the Verify arm forwarding the exact output"),
     ("featfix.py", "return float(np.abs(hd - hf).sum() / (np.abs(hf).sum() + EPS))",

@@ -537,6 +537,27 @@ def test_all_refresh_schedule_is_vanilla_bitwise():
     assert ca["refresh_steps"] == cb["refresh_steps"] == wl.steps
 
 
+def test_identity_blocks_make_every_arm_vanilla_bitwise():
+    """With every block the identity (both gates zero), the residual
+    increments a refresh stores are exactly zero, so every draft is exactly
+    its incoming state and every arm reproduces vanilla sampling bit for bit;
+    forecasting the block outputs themselves instead of their increments
+    (reading 1) would not."""
+    wl, sh, W, cond, xT = tiny_setup()
+    C = sh.hidden
+    W = dict(W)
+    for name in list(W):
+        if name.startswith("blk") and (name.endswith("mod.w") or name.endswith("mod.b")):
+            W[name] = W[name].copy()
+            W[name][2 * C:3 * C] = 0.0
+            W[name][5 * C:6 * C] = 0.0
+    ref, _, _ = featfix.run(W, sh, cond, xT, wl.steps, wl.refresh, wl.K, wl.sites, "vanilla")
+    for mode in ("featfix", "verify"):
+        x, logs, _ = featfix.run(W, sh, cond, xT, wl.steps, wl.refresh, wl.K, wl.sites, mode)
+        np.testing.assert_array_equal(x, ref)
+        assert all(g["rel_l1"] == 0.0 and g["rel_l2"] == 0.0 for g in logs)
+
+
 def test_featfix_site_forwards_the_exact_output():
     wl, sh, W, cond, xT = tiny_setup()
     seen = []
