@@ -27,7 +27,9 @@ Faster Cached Diffusion Inference"):
 Parity status: the method is an approximation (draft + sparse exact
 correction), so the oracle runs the algorithm step by step.  Its parts are
 pinned by ``tests/test_oracle_pins.py`` against closed forms, library
-routines, brute force and the paper's stated invariants.  Absolute latents on
+routines, brute force and the paper's stated invariants, and
+``tests/test_oracle_mutations.py`` plants plausible mistakes in a temporary
+copy of this package to show that a pin fails for each.  Absolute latents on
 random weights have no printed value in the paper: that end-to-end value is
 "parity unpinned" against the paper and is checked oracle <-> GPU only.
 """
