@@ -76,10 +76,14 @@ enum { FEATFIX_PLAN_EXACT = 0, FEATFIX_PLAN_DRAFT = 1, FEATFIX_PLAN_SITE = 2 };
  * input is the previous block's output, so the per-block increments
  * telescope, sum_l R_l = x_L - x_0; the forecast of the whole step is then
  * x_0 + sum_j w_j (x_L - x_0)_{s_j}, the same value as chaining the L
- * per-block drafts (up to rounding).  In the Verify arm every drafted step
- * is evaluated this way (so its forwarded trajectory is the one without
- * sites) and the paid check runs on a shadow copy that chains the per-block
- * drafts up to the site.  Steps with a debug capture always run per block. */
+ * per-block drafts (up to rounding).  A step with a FeatFix/Exact-only site
+ * drafts each run of consecutive drafted blocks (before, between and after
+ * its sites) in one pass: x + sum over the run's blocks of sum_j w_j R_j,
+ * read and written once.  In the Verify arm every drafted step is evaluated
+ * by the whole-step form (so its forwarded trajectory is the one without
+ * sites) and the paid checks run on a shadow copy drafted run by run up to
+ * the step's last site.  The flag restores one draft per block everywhere;
+ * steps with a debug capture always run per block. */
 #define FEATFIX_FLAG_PER_BLOCK_DRAFT 2u
 /* SITE_UPDATES_HISTORY takes the other reading of where the finite
  * differences of Eq. 2 are estimated: a site's exact increment h^f - u
