@@ -118,29 +118,47 @@ def _run_pins(tmp, select):
     return subprocess.run(cmd, cwd=tmp, env=env, capture_output=True, text=True, timeout=600)
 
 
-@pytest.fixture(scope="module")
-def pristine(tmp_path_factory):
-    tmp = str(tmp_path_factory.mktemp("oracle_copy"))
-    _copy(tmp)
-    return tmp
-
-
-def test_unmodified_copy_passes(pristine):
-    r = _run_pins(pristine, None)
-    assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-3000:]
-
-
-@pytest.mark.parametrize("fname,old,new,select,what", MUTATIONS, ids=[m[4] for m in MUTATIONS])
-def test_planted_mistake_fails_a_pin(tmp_path, fname, old, new, select, what):
-    tmp = str(tmp_path)
+def _mutant_run(case, tmp):
+    fname, old, new, select, what = case
     _copy(tmp)
     path = os.path.join(tmp, "oracle", fname)
     with open(path) as f:
         src = f.read()
-    assert src.count(old) == 1, "the text to change must occur once in oracle/%s" % fname
+    if src.count(old) != 1:
+        return None, "the text to change must occur once in oracle/%s" % fname
     with open(path, "w") as f:
         f.write(src.replace(old, new))
     r = _run_pins(tmp, select)
-    out = r.stdout + r.stderr
+    return r.returncode, r.stdout + r.stderr
+
+
+@pytest.fixture(scope="module")
+def runs(tmp_path_factory):
+    """The unmodified copy and every mutant, run four at a time."""
+    import concurrent.futures
+    cases = [None] + MUTATIONS
+    dirs = [str(tmp_path_factory.mktemp("oracle_copy")) for _ in cases]
+
+    def one(k):
+        if cases[k] is None:
+            _copy(dirs[k])
+            r = _run_pins(dirs[k], None)
+            return r.returncode, r.stdout + r.stderr
+        return _mutant_run(cases[k], dirs[k])
+
+    with concurrent.futures.ThreadPoolExecutor(max_workers=4) as ex:
+        res = list(ex.map(one, range(len(cases))))
+    return {"pristine": res[0], **{m[4]: res[k + 1] for k, m in enumerate(MUTATIONS)}}
+
+
+def test_unmodified_copy_passes(runs):
+    rc, out = runs["pristine"]
+    assert rc == 0, out[-6000:]
+
+
+@pytest.mark.parametrize("what", [m[4] for m in MUTATIONS])
+def test_planted_mistake_fails_a_pin(runs, what):
+    rc, out = runs[what]
+    assert rc is not None, out
     assert "no tests ran" not in out, out[-2000:]
-    assert r.returncode == 1, "%s: no pin failed\n%s" % (what, out[-3000:])
+    assert rc == 1, "%s: no pin failed\n%s" % (what, out[-3000:])
